@@ -1,0 +1,360 @@
+// Memory- and latency-bound kernels of the hot path:
+//   rmsnorm          pre-attention / pre-MLP normalisation (one warp per row)
+//   snr_scan         Seer Sec. 3.3 boundary criterion, one warp per sequence
+//   pack_route       Seer Sec. 3.4-3.5: micro-bucket routing (Eq. 4) fused
+//                    with device-resident compaction and the pinned control word
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace seer {
+namespace {
+
+// ------------------------------------------------------------------ RMSNorm
+template <int T>
+__device__ __forceinline__ void load8(const void* base, size_t i8, float (&v)[8]) {
+  if (T == kF32) {
+    const float4* p = reinterpret_cast<const float4*>(base) + 2 * i8;
+    const float4 a = p[0], b = p[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  } else {
+    const uint4 q = reinterpret_cast<const uint4*>(base)[i8];
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      v[2 * i] = lo16(w[i], T == kF16);
+      v[2 * i + 1] = hi16(w[i], T == kF16);
+    }
+  }
+}
+template <int T>
+__device__ __forceinline__ void store8(void* base, size_t i8, const float (&v)[8]) {
+  if (T == kF32) {
+    float4* p = reinterpret_cast<float4*>(base) + 2 * i8;
+    p[0] = make_float4(v[0], v[1], v[2], v[3]);
+    p[1] = make_float4(v[4], v[5], v[6], v[7]);
+  } else {
+    reinterpret_cast<uint4*>(base)[i8] =
+        make_uint4(pack2(v[0], v[1], T == kF16), pack2(v[2], v[3], T == kF16), pack2(v[4], v[5], T == kF16),
+                   pack2(v[6], v[7], T == kF16));
+  }
+}
+
+// y = x * rsqrt(mean(x^2) + eps) * g, one warp per row; input type IN, output
+// (and gain) type OUT; fp32 arithmetic.
+template <int IN, int OUT>
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ x, const void* __restrict__ g,
+                                                      void* __restrict__ y, int M_cap, const int* M_dev, int d,
+                                                      float eps, int* err) {
+  int M = M_cap;
+  if (M_dev != nullptr) {
+    const int md = *M_dev;
+    if (md < 0 || md > M_cap) {
+      if (blockIdx.x == 0 && threadIdx.x == 0) record_error(err, kErrRows);
+      M = md < 0 ? 0 : M_cap;
+    } else {
+      M = md;
+    }
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nwarps = gridDim.x * 8;
+  const int d8 = d / 8;
+  for (int row = blockIdx.x * 8 + warp; row < M; row += nwarps) {
+    const size_t base8 = static_cast<size_t>(row) * d8;
+    float ss = 0.f;
+    for (int v = lane; v < d8; v += 32) {
+      float e[8];
+      load8<IN>(x, base8 + v, e);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ss = fmaf(e[i], e[i], ss);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+    const float inv = rsqrtf(ss / static_cast<float>(d) + eps);
+    for (int v = lane; v < d8; v += 32) {
+      float e[8], gg[8];
+      load8<IN>(x, base8 + v, e);
+      load8<OUT>(g, v, gg);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) e[i] = e[i] * inv * gg[i];
+      store8<OUT>(y, base8 + v, e);
+    }
+  }
+}
+
+// Element-wise storage conversion (used once per model for f16 weight copies).
+template <int IN, int OUT>
+__global__ void convert_kernel(const void* __restrict__ src, void* __restrict__ dst, size_t n8) {
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n8;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    float e[8];
+    load8<IN>(src, i, e);
+    store8<OUT>(dst, i, e);
+  }
+}
+
+// ------------------------------------------------------------------ SNR scan
+// Sec. 3.3: first 0-based i in [1, N-w] with
+//   jump  = min(s_i .. s_{i+w-1}) - s_{i-1} >= tau_jump
+//   noise = max(s_i .. s_{i+w-1}) - min(..)  <= gamma * jump,   s = c / F,
+// evaluated in IEEE fp64 with explicit round-to-nearest operations (no FMA
+// contraction) so the decision is exactly reproducible.  L* = i* + 1, or N.
+__global__ void __launch_bounds__(32) snr_scan_kernel(const int* __restrict__ counts, int N, int F, double tau_jump,
+                                                      double gamma, int window, int* __restrict__ L_star,
+                                                      int* __restrict__ i_star) {
+  const int b = blockIdx.x;
+  const int lane = threadIdx.x;
+  const int* c = counts + static_cast<size_t>(b) * N;
+  const double Fd = static_cast<double>(F);
+  int found = -1;
+  const int last = N - window;   // inclusive
+  for (int base = 1; base <= last; base += 32) {
+    const int i = base + lane;
+    bool hit = false;
+    if (i <= last) {
+      int lo = c[i], hi = c[i];
+      for (int k = 1; k < window; ++k) {
+        const int v = c[i + k];
+        lo = min(lo, v);
+        hi = max(hi, v);
+      }
+      const double s_lo = __ddiv_rn(static_cast<double>(lo), Fd);
+      const double s_hi = __ddiv_rn(static_cast<double>(hi), Fd);
+      const double s_prev = __ddiv_rn(static_cast<double>(c[i - 1]), Fd);
+      const double jump = __dsub_rn(s_lo, s_prev);
+      const double noise = __dsub_rn(s_hi, s_lo);
+      hit = (jump >= tau_jump) && (noise <= __dmul_rn(gamma, jump));
+    }
+    const unsigned mask = __ballot_sync(0xffffffffu, hit);
+    if (mask) {
+      found = base + __ffs(mask) - 1;
+      break;
+    }
+  }
+  if (lane == 0) {
+    L_star[b] = found >= 0 ? found + 1 : N;
+    if (i_star) i_star[b] = found;
+  }
+}
+
+// ------------------------------------------------------------------ route + pack
+struct RouteSmem {
+  int n_buckets;
+  int bucket[kCtrlMaxGroups];
+  int count[kCtrlMaxGroups];
+  long long sum[kCtrlMaxGroups];
+  int path[kCtrlMaxGroups];
+  int rho_ppm[kCtrlMaxGroups];
+  int total, max_seg, pad_rows, path_mask, n_groups;
+};
+
+__device__ __forceinline__ int graph_capacity(int total) {
+  // smallest m * 2^e >= total with m in [8, 15]
+  if (total <= 8) return 8;
+  int e = 0;
+  while ((15 << e) < total) ++e;
+  const int m = (total + (1 << e) - 1) >> e;
+  return m << e;
+}
+
+// Every block recomputes the (tiny) routing decision in shared memory, block 0
+// publishes it, then all blocks copy rows.  Dynamic smem: seg/cu/bucket-index
+// arrays of B+1 ints each.
+__global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restrict__ x_full, int row_bytes,
+                                                         const int* __restrict__ cu_full,
+                                                         const int* __restrict__ ctx_len,
+                                                         const int* __restrict__ L_star, int B, int N, int T_cap,
+                                                         double tau_pad, int eager_max_bucket,
+                                                         uint8_t* __restrict__ x_packed, int* cu_out, int* kv_out,
+                                                         int* meta_out, int* host_ctrl, int epoch, int* err) {
+  extern __shared__ int dyn[];
+  int* seg = dyn;              // [B]
+  int* cus = dyn + B;          // [B+1]
+  int* bidx = dyn + 2 * B + 1; // [B]
+  __shared__ RouteSmem rs;
+
+  if (threadIdx.x == 0) {
+    int nb = 0;
+    for (int b = 8; b < N && nb < kCtrlMaxGroups - 1; b *= 2) rs.bucket[nb++] = b;
+    rs.bucket[nb++] = N;
+    rs.n_buckets = nb;
+    for (int k = 0; k < nb; ++k) { rs.count[k] = 0; rs.sum[k] = 0; }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < B; i += blockDim.x) {
+    int Ls = L_star[i];
+    if (Ls < 1 || Ls > N) {
+      if (blockIdx.x == 0) record_error(err, kErrBoundary);
+      Ls = Ls < 1 ? 1 : N;
+    }
+    int k = 0;
+    while (k < rs.n_buckets - 1 && Ls > rs.bucket[k]) ++k;
+    bidx[i] = k;
+    atomicAdd(&rs.count[k], 1);
+    atomicAdd(reinterpret_cast<unsigned long long*>(&rs.sum[k]), static_cast<unsigned long long>(Ls));
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int mask = 0, ng = 0;
+    for (int k = 0; k < rs.n_buckets; ++k) {
+      if (rs.count[k] == 0) { rs.path[k] = -1; continue; }
+      // Eq. 4, in fp64 exactly as written
+      const double rho = 1.0 - static_cast<double>(rs.sum[k]) / static_cast<double>(static_cast<long long>(rs.count[k]) * rs.bucket[k]);
+      int path;
+      if (rs.bucket[k] <= eager_max_bucket || rs.count[k] == 1) path = 2;
+      else if (rho <= tau_pad) path = 0;
+      else path = 1;
+      rs.path[k] = path;
+      rs.rho_ppm[k] = static_cast<int>(floor(rho * 1e6));
+      mask |= 1 << path;
+      ++ng;
+    }
+    rs.path_mask = mask;
+    rs.n_groups = ng;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < B; i += blockDim.x) {
+    int Ls = L_star[i];
+    Ls = Ls < 1 ? 1 : (Ls > N ? N : Ls);
+    const int k = bidx[i];
+    const int keep = rs.path[k] == 0 ? rs.bucket[k] : Ls;
+    const int ctx = ctx_len[i];
+    const int avail = cu_full[i + 1] - cu_full[i];
+    if (ctx < 0 || ctx + N > avail) {
+      if (blockIdx.x == 0) record_error(err, kErrLayout);
+    }
+    seg[i] = max(0, min(ctx + keep, avail));
+    if (blockIdx.x == 0) kv_out[i] = max(0, min(ctx + Ls, avail));
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0, mx = 0, pad = 0;
+    for (int i = 0; i < B; ++i) {
+      cus[i] = acc;
+      acc += seg[i];
+      mx = max(mx, seg[i]);
+      int Ls = L_star[i];
+      Ls = Ls < 1 ? 1 : (Ls > N ? N : Ls);
+      if (rs.path[bidx[i]] == 0) pad += rs.bucket[bidx[i]] - Ls;
+    }
+    cus[B] = acc;
+    rs.total = acc;
+    rs.max_seg = mx;
+    rs.pad_rows = pad;
+    if (acc > T_cap && blockIdx.x == 0) record_error(err, kErrCapacity);
+  }
+  __syncthreads();
+
+  if (blockIdx.x == 0) {
+    for (int i = threadIdx.x; i <= B; i += blockDim.x) cu_out[i] = cus[i];
+    if (threadIdx.x == 0) {
+      int w[kCtrlWords];
+      for (int i = 0; i < kCtrlWords; ++i) w[i] = 0;
+      w[1] = rs.total;
+      w[2] = rs.max_seg;
+      w[3] = graph_capacity(rs.total);
+      w[4] = rs.n_groups;
+      w[5] = rs.path_mask;
+      w[6] = rs.pad_rows;
+      int g = 0;
+      for (int k = 0; k < rs.n_buckets && g < kCtrlMaxGroups; ++k) {
+        if (rs.count[k] == 0) continue;
+        w[8 + 4 * g + 0] = rs.bucket[k];
+        w[8 + 4 * g + 1] = rs.count[k];
+        w[8 + 4 * g + 2] = rs.path[k];
+        w[8 + 4 * g + 3] = rs.rho_ppm[k];
+        ++g;
+      }
+      w[0] = epoch;
+      for (int i = 0; i < kCtrlWords; ++i) meta_out[i] = w[i];
+      if (host_ctrl != nullptr) {
+        volatile int* hc = host_ctrl;
+        for (int i = 1; i < kCtrlWords; ++i) hc[i] = w[i];
+        __threadfence_system();
+        hc[0] = epoch;
+        __threadfence_system();
+      }
+    }
+  }
+
+  // ---- copy rows, one warp per row, 16-byte vectors
+  const int total = min(rs.total, T_cap);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int vec = row_bytes / 16;
+  for (int r = blockIdx.x * 8 + warp; r < total; r += gridDim.x * 8) {
+    int lo = 0, hi = B;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (cus[mid] <= r) lo = mid; else hi = mid;
+    }
+    const int src = cu_full[lo] + (r - cus[lo]);
+    const uint4* s = reinterpret_cast<const uint4*>(x_full + static_cast<size_t>(src) * row_bytes);
+    uint4* dst = reinterpret_cast<uint4*>(x_packed + static_cast<size_t>(r) * row_bytes);
+    for (int v = lane; v < vec; v += 32) dst[v] = s[v];
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_rmsnorm(const void* x, int in_type, const void* g, void* y, int out_type, int M_cap,
+                           const int* M_dev, int d, float eps, int* err, cudaStream_t st) {
+  if (M_cap <= 0) return cudaSuccess;
+  int blocks = (M_cap + 7) / 8;
+  if (blocks > 65535 * 4) blocks = 65535 * 4;
+#define SEER_NORM(I, O) \
+  if (in_type == I && out_type == O) { rmsnorm_kernel<I, O><<<blocks, 256, 0, st>>>(x, g, y, M_cap, M_dev, d, eps, err); return cudaGetLastError(); }
+  SEER_NORM(kBF16, kF16)
+  SEER_NORM(kF16, kF16)
+  SEER_NORM(kBF16, kBF16)
+  SEER_NORM(kF32, kF32)
+#undef SEER_NORM
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  if (n % 8 != 0) return cudaErrorInvalidValue;
+  const size_t n8 = n / 8;
+  const int blocks = static_cast<int>(n8 / 256 + 1 < 4096 ? n8 / 256 + 1 : 4096);
+#define SEER_CONV(I, O) \
+  if (in_type == I && out_type == O) { convert_kernel<I, O><<<blocks, 256, 0, st>>>(src, dst, n8); return cudaGetLastError(); }
+  SEER_CONV(kBF16, kF16)
+  SEER_CONV(kF16, kBF16)
+  SEER_CONV(kBF16, kF32)
+  SEER_CONV(kF16, kF32)
+  SEER_CONV(kF32, kBF16)
+  SEER_CONV(kF32, kF16)
+#undef SEER_CONV
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,
+                            int* L_star, int* i_star, cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  snr_scan_kernel<<<B, 32, 0, st>>>(counts, N, F, tau_jump, gamma, window, L_star, i_star);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_full, const int* ctx_len,
+                              const int* L_star, int B, int d, int N, int T_cap, double tau_pad,
+                              int eager_max_bucket, void* x_packed, int* cu_out, int* kv_out, int* meta_out,
+                              int* host_ctrl_dev, int epoch, int* err, int num_sms, cudaStream_t st) {
+  const size_t sm = static_cast<size_t>(3 * B + 1) * sizeof(int);
+  if (sm > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(pack_route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(sm));
+    if (e != cudaSuccess) return e;
+  }
+  int blocks = (T_cap + 7) / 8;
+  const int cap = num_sms * 8;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  pack_route_kernel<<<blocks, 256, sm, st>>>(reinterpret_cast<const uint8_t*>(x_full), d * elem_bytes, cu_full,
+                                             ctx_len, L_star, B, N, T_cap, tau_pad, eager_max_bucket,
+                                             reinterpret_cast<uint8_t*>(x_packed), cu_out, kv_out, meta_out,
+                                             host_ctrl_dev, epoch, err);
+  return cudaGetLastError();
+}
+
+}  // namespace seer

@@ -1,0 +1,83 @@
+// Internal launch interface between the C-ABI layer (seer_api.cu) and the
+// kernel translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace seer {
+
+// Epilogue variants of the GEMM kernels.
+enum GemmMode : int {
+  kGemmStore = 0,     // C = A B^T
+  kGemmResidual = 1,  // C = A B^T + R
+  kGemmSwiglu = 2,    // act = SiLU(A Bg^T) * (A Bu^T), optional near-zero counts
+  kGemmCount = 3,     // counts only (detector): A rows gathered per sequence window
+};
+
+struct GemmParams {
+  int M_cap;              // rows available in A / C
+  const int* M_dev;       // optional device row count (<= M_cap)
+  int N;                  // output columns (Swiglu/Count: F)
+  int K;
+  void* C;                // output [M, ldc]
+  int ldc;
+  const void* R;          // residual [M, ldr]
+  int ldr;
+  int* counts;            // [B * Nw] near-zero counts (Swiglu hook / Count)
+  float act_eps;
+  const int* cu;          // segment offsets [B+1] for the Swiglu count hook
+  int B;
+  const int* resp_start;  // first response row per sequence
+  int Nw;                 // response window
+  int* err;               // device error word
+  uint32_t idesc;         // tcgen05 instruction descriptor (operand type f16 or bf16)
+  int out_type;           // ElemType of C (kBF16 / kF16; kF32 on the CUDA-core path)
+  int res_type;           // ElemType of R
+};
+
+struct AttnParams {
+  const int* cu;          // [B+1]
+  const int* kv_len;      // [B] or null
+  int B;
+  int T_cap;
+  int n_heads;
+  int head_dim;
+  void* out;              // [T, H*dh]
+  int ldo;                // elements
+  const int4* work;       // schedule: (b, h, q-tile, 0)
+  const int* work_count;
+  int* err;
+};
+
+// tcgen05 / TMA kernels (16-bit operands).  Tensor maps are encoded on the host.
+int tc_gemm_smem_bytes();
+cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
+                           const GemmParams& p, int num_sms, cudaStream_t st);
+int tc_attn_smem_bytes();
+cudaError_t launch_tc_attn(const CUtensorMap& mQKV, const AttnParams& p, int grid, bool f16, cudaStream_t st);
+cudaError_t launch_attn_schedule(const int* cu, const int* kv_len, int B, int n_heads, int T_cap, int4* work,
+                                 int* work_count, int max_units, int* err, cudaStream_t st);
+
+// CUDA-core kernels (fp32 storage; small shapes).
+cudaError_t launch_simt_gemm(int mode, const float* A, const float* B0, const float* B1, const GemmParams& p,
+                             cudaStream_t st);
+cudaError_t launch_simt_attn(const float* qkv, const AttnParams& p, cudaStream_t st);
+
+// Element-wise / scan kernels (both storage types).
+cudaError_t launch_rmsnorm(const void* x, int in_type, const void* g, void* y, int out_type, int M_cap,
+                           const int* M_dev, int d, float eps, int* err, cudaStream_t st);
+cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, cudaStream_t st);
+cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,
+                            int* L_star, int* i_star, cudaStream_t st);
+cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_full, const int* ctx_len,
+                              const int* L_star, int B, int d, int N, int T_cap, double tau_pad,
+                              int eager_max_bucket, void* x_packed, int* cu_out, int* kv_out, int* meta_out,
+                              int* host_ctrl_dev, int epoch, int* err, int num_sms, cudaStream_t st);
+
+constexpr int kCtrlMaxGroups = 32;
+constexpr int kCtrlWords = 8 + 4 * kCtrlMaxGroups;
+
+}  // namespace seer

@@ -1,0 +1,338 @@
+// Persistent tcgen05 GEMM for sm_103a: C[M, N] = A[M, K] * B[N, K]^T with
+// 16-bit operands (both f16 or both bf16, chosen by the instruction
+// descriptor) and fp32 accumulation in tensor memory (TMEM); C and the
+// residual R are f16 or bf16 independently.
+//
+// One CTA per SM, 192 threads, warp-specialised:
+//   warp 0      TMA producer: 128x64 A tile + two 128x64 B tiles per stage
+//               (128-byte swizzle), 4-stage ring of 48 KB stages;
+//   warp 1      TMEM allocator + single-thread MMA issuer: 4 x
+//               tcgen05.mma (M=128, N=256, K=16) per stage into one of two
+//               256-column fp32 accumulators (double buffered, 512 columns);
+//   warps 2-5   epilogue: tcgen05.ld of the accumulator (each warp owns one
+//               32-lane quarter of TMEM = 32 output rows), fused epilogue,
+//               16-byte global stores.
+// The epilogue of tile t overlaps the main loop of tile t+1.
+//
+// Epilogues (Sec. 3.1 Eq. 2 projections; Sec. 3.2 sparsity hook):
+//   Store     C = A B^T                                    (QKV projection)
+//   Residual  C = A B^T + R                                (O / down projection)
+//   Swiglu    B = [Wg tile ; Wu tile] -> act = SiLU(g) * u  (gate/up), plus the
+//             per-row count of |act| < eps on response rows (step-0 hook)
+//   Count     detector: A rows gathered per sequence window, counts only
+#include "common.cuh"
+#include "kernels.h"
+
+namespace seer {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 64;
+constexpr int STAGES = 4;
+constexpr int A_TILE_BYTES = BM * BK * 2;            // 16 KB
+constexpr int B_HALF_BYTES = 128 * BK * 2;           // 16 KB
+constexpr int STAGE_BYTES = A_TILE_BYTES + 2 * B_HALF_BYTES;  // 48 KB
+constexpr int THREADS = 192;
+constexpr int ACC_COLS = 256;
+constexpr int TMEM_COLS = 512;
+constexpr int GROUP_M = 16;                          // m-tiles per raster group (L2 reuse)
+constexpr int BAR_BYTES = 256;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
+
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int& m, int& n) {
+  const int per_group = GROUP_M * num_n;
+  const int g = t / per_group;
+  const int r = t - g * per_group;
+  const int m0 = g * GROUP_M;
+  const int gm = min(GROUP_M, num_m - m0);
+  m = m0 + r % gm;
+  n = r / gm;
+}
+
+__device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)); }
+
+template <int MODE>
+__global__ void __launch_bounds__(THREADS, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB0,
+                   const __grid_constant__ CUtensorMap mB1, const GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* acc_full = empty + STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  // ---- problem size (device row counts are clamped, never trusted blindly)
+  int M = p.M_cap;
+  int num_m, tiles_per_seq = 1;
+  if (MODE == kGemmCount) {
+    tiles_per_seq = (p.Nw + BM - 1) / BM;
+    num_m = p.B * tiles_per_seq;
+  } else {
+    if (p.M_dev != nullptr) {
+      const int md = *p.M_dev;
+      if (md < 0 || md > p.M_cap) {
+        if (threadIdx.x == 0 && blockIdx.x == 0) record_error(p.err, kErrRows);
+        M = md < 0 ? 0 : p.M_cap;
+      } else {
+        M = md;
+      }
+    }
+    num_m = (M + BM - 1) / BM;
+  }
+  const bool halfN = (MODE == kGemmSwiglu || MODE == kGemmCount);
+  const int num_n = halfN ? p.N / 128 : p.N / BN;
+  const int num_tiles = num_m * num_n;
+  const int KB = p.K / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], 4);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      tma_prefetch_desc(&mA);
+      tma_prefetch_desc(&mB0);
+      tma_prefetch_desc(&mB1);
+      int s = 0;
+      uint32_t ph = 0;
+      long issued = 0;
+      for (int t = blockIdx.x; t < num_tiles && !*abort_flag; t += gridDim.x) {
+        int m, n;
+        tile_coords(t, num_m, num_n, m, n);
+        int a_row;
+        if (MODE == kGemmCount) {
+          const int b = m / tiles_per_seq;
+          const int j = m - b * tiles_per_seq;
+          const int rs = p.resp_start[b];
+          if (rs < 0 || rs + p.Nw > p.M_cap) record_error(p.err, kErrLayout);
+          a_row = rs + j * BM;
+        } else {
+          a_row = m * BM;
+        }
+        const int b_row0 = halfN ? n * 128 : n * BN;
+        const int b_row1 = halfN ? n * 128 : n * BN + 128;
+        bool ok = true;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.err)) { ok = false; break; }
+          uint8_t* sa = smem + s * STAGE_BYTES;
+          mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
+          tma_load_2d(sa, &mA, &full[s], kb * BK, a_row);
+          tma_load_2d(sa + A_TILE_BYTES, &mB0, &full[s], kb * BK, b_row0);
+          tma_load_2d(sa + A_TILE_BYTES + B_HALF_BYTES, &mB1, &full[s], kb * BK, b_row1);
+          ++issued;
+          if (++s == STAGES) { s = 0; ph ^= 1u; }
+        }
+        if (!ok) break;
+      }
+      if (*abort_flag) {
+        // let copies still in flight land before the CTA's shared memory is released
+        const long first = issued > STAGES ? issued - STAGES : 0;
+        for (long i = first; i < issued; ++i)
+          mbar_wait_drain(&full[i % STAGES], static_cast<uint32_t>((i / STAGES) & 1), 200000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      const uint32_t idesc = p.idesc;
+      int s = 0;
+      uint32_t ph = 0;
+      int acc = 0;
+      uint32_t acc_ph = 0;
+      for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+        if (!mbar_wait(&acc_empty[acc], acc_ph ^ 1u, abort_flag, p.err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * ACC_COLS);
+        bool ok = true;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&full[s], ph, abort_flag, p.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
+          const uint64_t adesc = make_sdesc_sw128(sa, 16, 1024);
+          const uint64_t bdesc = make_sdesc_sw128(sa + A_TILE_BYTES, 16, 1024);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            // +32 bytes along K inside the 128-byte swizzle atom = +2 in the address field
+            tc_mma_f16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
+          }
+          tc_commit(&empty[s]);
+          if (++s == STAGES) { s = 0; ph ^= 1u; }
+        }
+        if (!ok) break;
+        tc_commit(&acc_full[acc]);
+        if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
+      }
+    }
+  } else {
+    // -------------------------------------------------- epilogue warps 2..5
+    const int q = warp & 3;                    // TMEM lane quarter owned by this warp
+    const int row_in_tile = q * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+      int m, n;
+      tile_coords(t, num_m, num_n, m, n);
+      if (!mbar_wait(&acc_full[acc], acc_ph, abort_flag, p.err)) break;
+      tc_fence_after();
+      const uint32_t tacc = tmem_base + lane_off + static_cast<uint32_t>(acc * ACC_COLS);
+      if (MODE == kGemmStore || MODE == kGemmResidual) {
+        const int row = m * BM + row_in_tile;
+        const bool valid = row < M;
+        const bool of16 = p.out_type == kF16, rf16 = p.res_type == kF16;
+        uint16_t* crow = reinterpret_cast<uint16_t*>(p.C) + static_cast<size_t>(valid ? row : 0) * p.ldc + n * BN;
+        const uint16_t* rrow =
+            MODE == kGemmResidual ? reinterpret_cast<const uint16_t*>(p.R) + static_cast<size_t>(valid ? row : 0) * p.ldr + n * BN
+                                  : nullptr;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tacc + c * 32, r);
+          tmem_ld_wait();
+          if (valid) {
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+            if (MODE == kGemmResidual) {
+              const uint4* rp = reinterpret_cast<const uint4*>(rrow + c * 32);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const uint4 rv = rp[i];
+                v[8 * i + 0] += lo16(rv.x, rf16); v[8 * i + 1] += hi16(rv.x, rf16);
+                v[8 * i + 2] += lo16(rv.y, rf16); v[8 * i + 3] += hi16(rv.y, rf16);
+                v[8 * i + 4] += lo16(rv.z, rf16); v[8 * i + 5] += hi16(rv.z, rf16);
+                v[8 * i + 6] += lo16(rv.w, rf16); v[8 * i + 7] += hi16(rv.w, rf16);
+              }
+            }
+            uint4* cp = reinterpret_cast<uint4*>(crow + c * 32);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              cp[i] = make_uint4(pack2(v[8 * i + 0], v[8 * i + 1], of16), pack2(v[8 * i + 2], v[8 * i + 3], of16),
+                                 pack2(v[8 * i + 4], v[8 * i + 5], of16), pack2(v[8 * i + 6], v[8 * i + 7], of16));
+            }
+          }
+        }
+      } else {
+        // gate columns 0..127, up columns 128..255 of the accumulator
+        int row, cnt_idx = -1;
+        bool store = false;
+        if (MODE == kGemmCount) {
+          const int b = m / tiles_per_seq;
+          const int tl = (m - b * tiles_per_seq) * BM + row_in_tile;
+          row = -1;
+          if (tl < p.Nw) cnt_idx = b * p.Nw + tl;
+        } else {
+          row = m * BM + row_in_tile;
+          store = row < M;
+          if (store && p.counts != nullptr) {
+            // segment of this row (binary search in cu), then its window offset
+            int lo = 0, hi = p.B;
+            while (hi - lo > 1) {
+              const int mid = (lo + hi) >> 1;
+              if (p.cu[mid] <= row) lo = mid; else hi = mid;
+            }
+            const int tl = row - p.resp_start[lo];
+            if (tl >= 0 && tl < p.Nw && row < p.cu[lo + 1]) cnt_idx = lo * p.Nw + tl;
+          }
+        }
+        int cnt = 0;
+        const bool of16 = p.out_type == kF16;
+        uint16_t* arow =
+            MODE == kGemmSwiglu ? reinterpret_cast<uint16_t*>(p.C) + static_cast<size_t>(store ? row : 0) * p.ldc + n * 128
+                                : nullptr;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t g[32], u[32];
+          tmem_ld32(tacc + c * 32, g);
+          tmem_ld32(tacc + 128 + c * 32, u);
+          tmem_ld_wait();
+          float a[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            a[i] = silu_f(__uint_as_float(g[i])) * __uint_as_float(u[i]);
+            cnt += fabsf(a[i]) < p.act_eps ? 1 : 0;
+          }
+          if (MODE == kGemmSwiglu && store) {
+            uint4* cp = reinterpret_cast<uint4*>(arow + c * 32);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              cp[i] = make_uint4(pack2(a[8 * i + 0], a[8 * i + 1], of16), pack2(a[8 * i + 2], a[8 * i + 3], of16),
+                                 pack2(a[8 * i + 4], a[8 * i + 5], of16), pack2(a[8 * i + 6], a[8 * i + 7], of16));
+            }
+          }
+        }
+        if (cnt_idx >= 0 && p.counts != nullptr) atomicAdd(&p.counts[cnt_idx], cnt);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[acc]);
+      if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+template <int MODE>
+cudaError_t launch_mode(const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1, const GemmParams& p,
+                        int num_sms, cudaStream_t st) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  long num_m;
+  if (MODE == kGemmCount) num_m = static_cast<long>(p.B) * ((p.Nw + BM - 1) / BM);
+  else num_m = (p.M_cap + BM - 1) / BM;
+  const long num_n = (MODE == kGemmSwiglu || MODE == kGemmCount) ? p.N / 128 : p.N / BN;
+  long tiles = num_m * num_n;
+  if (tiles <= 0) return cudaSuccess;
+  const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
+  tc_gemm_kernel<MODE><<<grid, THREADS, SMEM_BYTES, st>>>(mA, mB0, mB1, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int tc_gemm_smem_bytes() { return SMEM_BYTES; }
+
+cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
+                           const GemmParams& p, int num_sms, cudaStream_t st) {
+  switch (mode) {
+    case kGemmStore: return launch_mode<kGemmStore>(mA, mB0, mB1, p, num_sms, st);
+    case kGemmResidual: return launch_mode<kGemmResidual>(mA, mB0, mB1, p, num_sms, st);
+    case kGemmSwiglu: return launch_mode<kGemmSwiglu>(mA, mB0, mB1, p, num_sms, st);
+    case kGemmCount: return launch_mode<kGemmCount>(mA, mB0, mB1, p, num_sms, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace seer

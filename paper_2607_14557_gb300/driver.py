@@ -1,0 +1,199 @@
+"""One-GPU driver of the Seer hot path (argument marshalling and buffers only).
+
+The driver owns the device buffers of one batch and enqueues the library's
+entry points on one CUDA stream:
+
+* ``SeerPath.step`` -- the step-0 detector (Sec. 3.2-3.3), routing +
+  device-resident compaction (Sec. 3.4-3.5) and one truncated layer
+  (Sec. 3.6), all enqueued back to back with no host synchronisation: every
+  kernel reads the packed row count from device memory, so the layer can be
+  queued before the host has seen the route.  The host reads the route later
+  from the pinned control word (``SeerPath.route``), i.e. the latency of the
+  decision is hidden behind the GPU work ("latency shadowing").
+* ``SeerPath.padded_forward`` -- the same layer kernels over the untruncated
+  window (the comparator of the speedup).
+* ``SeerStack`` -- the multi-layer, multi-step denoising loop: one full
+  step-0 pass (counts fused into the detection layer's gate/up epilogue),
+  boundary scan and compaction, then the remaining steps over the packed
+  sequences, replayed from a CUDA graph captured per graph capacity.
+
+Every computation happens in libseer's CUDA kernels; this module never
+touches tensor values on the host.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict, List, Optional
+
+import numpy as np
+import torch
+
+from . import seer as S
+
+
+def _dev():
+    return torch.device("cuda", torch.cuda.current_device())
+
+
+def f16_copy(t: torch.Tensor) -> torch.Tensor:
+    """f16 copy of a bf16 device tensor made by the library's converter."""
+    dst = torch.empty(t.shape, dtype=torch.float16, device=t.device)
+    S.seer_convert(t, "bf16", dst, "f16", t.numel())
+    return dst
+
+
+@dataclasses.dataclass
+class LayerWeights:
+    """Device weights of one block.  ``model`` holds the model-dtype tensors
+    (the detector reads gate/up from here); ``run`` the tensors the layer
+    kernels read (f16 copies for a bf16 model)."""
+    model: Dict[str, torch.Tensor]
+    run: Dict[str, torch.Tensor]
+
+    @staticmethod
+    def from_host(w: Dict[str, np.ndarray], dtype: str, device=None) -> "LayerWeights":
+        device = device or _dev()
+        tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+        up = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(device=device, dtype=tdt)
+        model = {"w_qkv": up(np.concatenate([w["wq"], w["wk"], w["wv"]], axis=0)), "w_o": up(w["wo"]),
+                 "w_gate": up(w["wg"]), "w_up": up(w["wu"]), "w_down": up(w["wd"]), "g_attn": up(w["g_attn"]),
+                 "g_mlp": up(w["g_mlp"])}
+        run = model if dtype == "f32" else {k: f16_copy(v) for k, v in model.items()}
+        return LayerWeights(model, run)
+
+    def struct(self) -> S.seer_layer_weights:
+        r = self.run
+        return S.make_weights(r["w_qkv"], r["w_o"], r["w_gate"], r["w_up"], r["w_down"], r["g_attn"], r["g_mlp"])
+
+    def drop_model_copy(self, keep=("w_gate", "w_up")):
+        """Free the model-dtype tensors the kernels no longer need."""
+        if self.model is self.run:
+            return
+        self.model = {k: v for k, v in self.model.items() if k in keep}
+
+
+class SeerPath:
+    """Buffers and launches of one batch through detect -> pack -> layer."""
+
+    def __init__(self, dims: S.seer_dims, dtype: str, B: int, N: int, T_full: int, params: S.seer_params,
+                 device=None):
+        self.dims, self.dtype, self.B, self.N, self.T_full, self.params = dims, dtype, B, N, T_full, params
+        dev = self.device = device or _dev()
+        tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+        d = dims.d_model
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.counts = torch.empty(B * N, **i32)
+        self.L_star = torch.empty(B, **i32)
+        self.i_star = torch.empty(B, **i32)
+        self.cu = torch.empty(B + 1, **i32)
+        self.kv = torch.empty(B, **i32)
+        self.meta = torch.empty(S.CTRL_WORDS, **i32)
+        self.host_ctrl = torch.zeros(S.CTRL_WORDS, dtype=torch.int32).pin_memory()
+        self.ctrl = torch.zeros(S.CTRL_WORDS, dtype=torch.int32)
+        self.x_packed = torch.zeros((T_full, d), dtype=tdt, device=dev)
+        self.y = torch.empty((T_full, d), dtype=tdt, device=dev)
+        self.ws_bytes = S.seer_layer_workspace_size(dims, dtype, T_full, B)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=dev)
+        self.epoch = 0
+
+    def detect(self, x_full, resp_start, w: LayerWeights, stream=None):
+        S.seer_detect_boundary(x_full, self.dtype, x_full.shape[0], resp_start, self.B, self.N, w.model["w_gate"],
+                               w.model["w_up"], self.dims, self.params, self.counts, self.L_star, self.i_star,
+                               stream=stream)
+
+    def pack(self, x_full, cu_full, ctx_len, stream=None):
+        self.epoch += 1
+        S.seer_pack_ragged(x_full, self.dtype, cu_full, ctx_len, self.L_star, self.B, self.dims.d_model, self.N,
+                           self.T_full, self.params, self.x_packed, self.cu, self.kv, self.meta, self.host_ctrl,
+                           self.epoch, stream=stream)
+
+    def layer(self, w: LayerWeights, x=None, y=None, cu=None, kv=None, T_cap=None, stream=None):
+        x = self.x_packed if x is None else x
+        y = self.y if y is None else y
+        S.seer_layer_forward(w.struct(), self.dims, self.dtype, x, y, self.cu if cu is None else cu,
+                             self.kv if cu is None else kv, self.B, self.T_full if T_cap is None else T_cap, None, 0,
+                             0.0, None, self.ws, self.ws_bytes, stream=stream)
+
+    def step(self, x_full, cu_full, resp_start, ctx_len, w: LayerWeights, stream=None):
+        """Detect, route + pack and run the truncated layer; nothing waits on the host."""
+        self.detect(x_full, resp_start, w, stream)
+        self.pack(x_full, cu_full, ctx_len, stream)
+        self.layer(w, stream=stream)
+
+    def route(self, timeout_us: int = 10_000_000) -> Dict[str, object]:
+        """Read the route of the last pack from the pinned control word."""
+        S.seer_poll_ctrl(self.host_ctrl, self.epoch, timeout_us, self.ctrl)
+        c = self.ctrl.numpy()
+        groups = [{"bucket": int(c[8 + 4 * g]), "members": int(c[9 + 4 * g]), "path": int(c[10 + 4 * g]),
+                   "rho": c[11 + 4 * g] / 1e6} for g in range(int(c[4]))]
+        return {"total": int(c[1]), "max_seqlen": int(c[2]), "capacity": int(c[3]), "path_mask": int(c[5]),
+                "pad_rows": int(c[6]), "groups": groups}
+
+    def padded_forward(self, x_full, cu_full, w: LayerWeights, y_full, stream=None):
+        """The same layer over the untruncated windows (every key kept)."""
+        S.seer_layer_forward(w.struct(), self.dims, self.dtype, x_full, y_full, cu_full, None, self.B, self.T_full,
+                             None, 0, 0.0, None, self.ws, self.ws_bytes, stream=stream)
+
+
+class SeerStack:
+    """Denoising loop over a stack of layers (one GPU).
+
+    Step 0 runs every layer over the full windows; the detection layer's
+    gate/up epilogue counts near-zero activations of the response rows, the
+    SNR scan turns them into L*, and the fused route/pack kernel compacts the
+    step-0 *input* rows.  Steps 1..T-1 then run every layer over the packed
+    sequences.  The step body is captured once into a CUDA graph (kernels
+    read the packed row count from device memory, so the graph serves any
+    total up to the capacity) and replayed.
+    """
+
+    def __init__(self, dims, dtype, B, N, T_full, params, layers: List[LayerWeights], detect_layer: int = 3,
+                 device=None):
+        self.path = SeerPath(dims, dtype, B, N, T_full, params, device)
+        self.layers = layers
+        self.detect_layer = detect_layer
+        dev = self.path.device
+        tdt = self.path.x_packed.dtype
+        d = dims.d_model
+        self.buf = [torch.empty((T_full, d), dtype=tdt, device=dev) for _ in range(2)]
+        self.graphs: Dict[int, torch.cuda.CUDAGraph] = {}
+
+    def _run_layers(self, x, cu, kv, T_cap, resp_start=None, stream=None):
+        p = self.path
+        cur = x
+        for li, w in enumerate(self.layers):
+            out = self.buf[li % 2] if cur is not self.buf[li % 2] else self.buf[(li + 1) % 2]
+            count = resp_start is not None and li == self.detect_layer
+            S.seer_layer_forward(w.struct(), p.dims, p.dtype, cur, out, cu, kv, p.B, T_cap,
+                                 resp_start if count else None, p.N if count else 0,
+                                 p.params.act_eps if count else 0.0, p.counts if count else None, p.ws, p.ws_bytes,
+                                 stream=stream)
+            cur = out
+        return cur
+
+    def step0(self, x_full, cu_full, resp_start, ctx_len, stream=None):
+        """Full-window step with the fused detection hook, then scan + pack."""
+        p = self.path
+        self._run_layers(x_full, cu_full, None, p.T_full, resp_start=resp_start, stream=stream)
+        S.seer_snr_scan(p.counts, p.B, p.N, p.dims.d_ff, p.params, p.L_star, p.i_star, stream=stream)
+        p.pack(x_full, cu_full, ctx_len, stream)
+
+    def truncated_step(self, stream=None):
+        p = self.path
+        return self._run_layers(p.x_packed, p.cu, p.kv, p.T_full, stream=stream)
+
+    def padded_step(self, x_full, cu_full, stream=None):
+        return self._run_layers(x_full, cu_full, None, self.path.T_full, stream=stream)
+
+    def capture(self, fn, key):
+        """Capture ``fn`` (a step body) into a CUDA graph stored under ``key``."""
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            fn(stream=s)                       # warm-up outside capture
+        torch.cuda.current_stream().wait_stream(s)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            fn(stream=torch.cuda.current_stream())
+        self.graphs[key] = g
+        return g

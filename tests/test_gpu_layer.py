@@ -1,0 +1,137 @@
+"""GPU parity of the full path: detect (S1-S2) -> route + pack (S3-S4) ->
+truncated layer forward (S5-S11), through the C ABI, against the oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from tests.helpers import check_close, cuda, host, i32, layer_weight_tensors, to_dev, weights_struct
+
+pytestmark = pytest.mark.gpu
+
+S = pytest.importorskip("paper_2607_14557_gb300.seer")
+
+
+@pytest.fixture(autouse=True)
+def _device_clean():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    yield
+    assert S.seer_check_device() == 0
+
+
+def run_path(wl, lens=None, tau_pad=0.2, extra_cap=64, data=None):
+    """Detect, pack and run one layer on the GPU; return everything needed to check it."""
+    dt = wl.dtype
+    lens = lens or synth.lengths(wl)
+    x, cu_full, resp = data if data is not None else synth.hidden_full(wl, lens)
+    w = synth.layer_weights(wl, 0)
+    B, N, F, d = wl.batch, wl.window, wl.d_ff, wl.d
+    dims = S.make_dims(d, wl.n_heads, wl.head_dim, F)
+    params = S.make_params(wl.act_eps, tau_pad=tau_pad)
+    W, WL = layer_weight_tensors(wl, w)
+    xd = to_dev(x, dt)
+    counts = torch.empty(B * N, dtype=torch.int32, device=cuda())
+    L = torch.empty(B, dtype=torch.int32, device=cuda())
+    S.seer_detect_boundary(xd, dt, x.shape[0], i32(resp), B, N, W["w_gate"], W["w_up"], dims, params, counts, L)
+    T_cap = int(cu_full[-1]) + extra_cap
+    xp = torch.full((T_cap, d), 0.0, dtype=xd.dtype, device=cuda())
+    cu = torch.empty(B + 1, dtype=torch.int32, device=cuda())
+    kv = torch.empty(B, dtype=torch.int32, device=cuda())
+    meta = torch.empty(S.CTRL_WORDS, dtype=torch.int32, device=cuda())
+    S.seer_pack_ragged(xd, dt, i32(cu_full), i32(lens.ctx), L, B, d, N, T_cap, params, xp, cu, kv, meta)
+    y = torch.full((T_cap, d), 9.0, dtype=xd.dtype, device=cuda())
+    ws_bytes = S.seer_layer_workspace_size(dims, dt, T_cap, B)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=cuda())
+    S.seer_layer_forward(weights_struct(WL), dims, dt, xp, y, cu, kv, B, T_cap, None, 0, 0.0, None, ws, ws_bytes)
+    torch.cuda.synchronize()
+    return dict(x=x, cu_full=cu_full, resp=resp, w=w, lens=lens, counts=counts.cpu().numpy().reshape(B, N),
+                L=L.cpu().numpy(), cu=cu.cpu().numpy(), kv=kv.cpu().numpy(), xp=host(xp), y=host(y), T_cap=T_cap)
+
+
+def _check_path(wl, r):
+    lens = r["lens"]
+    np.testing.assert_array_equal(r["L"], lens.boundary + 1)           # planted boundary, bit exact
+    seg, kv, cu = oracle.segment_layout(lens.ctx, r["L"], wl.window)
+    np.testing.assert_array_equal(r["cu"], cu)
+    np.testing.assert_array_equal(r["kv"], kv)
+    T = int(cu[-1])
+    np.testing.assert_array_equal(r["xp"][:T], oracle.pack_rows(r["x"], r["cu_full"], seg))
+    ref = oracle.layer_forward_packed(r["xp"][:T], cu, r["w"], wl.n_heads, kv_len=kv)
+    err = check_close(r["y"][:T], ref, wl.dtype, wl.name)
+    assert (r["y"][T:] == 9.0).all()                                    # zero work past truncation
+    return err
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_tiny_bf16_path(seed):
+    wl = synth.tiny_workload(dtype="bf16", seed=300 + seed, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4,
+                             window=200, boundary=("uniform", 8, 190), visual=("mult", 96, 1, 3))
+    _check_path(wl, run_path(wl))
+
+
+def test_tiny_bf16_static_route_pads_and_masks():
+    # lengths concentrated in one bucket -> static path (padded rows are masked keys)
+    wl = synth.tiny_workload(dtype="bf16", seed=310, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4,
+                             window=200, boundary=("uniform", 120, 127))
+    r = run_path(wl)
+    groups = oracle.route(r["L"], wl.window)
+    assert any(g["path"] == oracle.PATH_STATIC for g in groups)
+    _check_path(wl, r)
+
+
+def test_workload0_f32_path():
+    wl = synth.workload(0)
+    _check_path(wl, run_path(wl))
+
+
+def test_workload1_bf16_path():
+    wl = synth.workload(1)
+    _check_path(wl, run_path(wl))
+
+
+def test_batch_permutation_is_bit_exact():
+    wl = synth.tiny_workload(dtype="bf16", seed=320, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4,
+                             window=160, boundary=("uniform", 8, 150))
+    lens = synth.lengths(wl)
+    r1 = run_path(wl, lens)
+    perm = np.array([2, 0, 3, 1])
+    x, cu_full = r1["x"], r1["cu_full"]
+    seqs = [x[cu_full[i]:cu_full[i + 1]] for i in range(wl.batch)]
+    lens_p = synth.with_lengths(wl, lens, visual=lens.visual[perm], prompt=lens.prompt[perm],
+                                boundary=lens.boundary[perm])
+    cuf = np.concatenate([[0], np.cumsum(lens_p.full)]).astype(np.int32)
+    data = (np.concatenate([seqs[i] for i in perm]), cuf, (cuf[:-1] + lens_p.ctx).astype(np.int32))
+    r2 = run_path(wl, lens_p, data=data)
+    for j, i in enumerate(perm):
+        a = r1["y"][r1["cu"][i]:r1["cu"][i + 1]]
+        b = r2["y"][r2["cu"][j]:r2["cu"][j + 1]]
+        np.testing.assert_array_equal(a, b)
+
+
+def test_layer_count_hook_on_full_window():
+    # step-0 style: full (untruncated) window, counts fused into the gate/up epilogue
+    wl = synth.tiny_workload(dtype="bf16", seed=330, d=256, n_heads=2, head_dim=128, d_ff=768, batch=3, window=160,
+                             boundary=("uniform", 8, 150))
+    lens = synth.lengths(wl)
+    x, cu_full, resp = synth.hidden_full(wl, lens)
+    w = synth.layer_weights(wl, 0)
+    B, N, F, d = wl.batch, wl.window, wl.d_ff, wl.d
+    dims = S.make_dims(d, wl.n_heads, wl.head_dim, F)
+    W, WL = layer_weight_tensors(wl, w)
+    T = x.shape[0]
+    y = torch.empty((T, d), dtype=torch.bfloat16, device=cuda())
+    counts = torch.full((B * N,), -1, dtype=torch.int32, device=cuda())
+    ws_bytes = S.seer_layer_workspace_size(dims, "bf16", T, B)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=cuda())
+    S.seer_layer_forward(weights_struct(WL), dims, "bf16", to_dev(x, "bf16"), y, i32(cu_full), None, B, T, i32(resp),
+                         N, 0.05, counts, ws, ws_bytes)
+    got = counts.cpu().numpy().reshape(B, N)
+    yh = host(y)
+    for b in range(B):
+        seg = x[cu_full[b]:cu_full[b + 1]]
+        rows = np.arange(resp[b] - cu_full[b], resp[b] - cu_full[b] + N)
+        parts = oracle.layer_forward_segment(seg, w, wl.n_heads, count_rows=rows, act_eps=0.05, return_parts=True)
+        assert np.abs(got[b] - parts["counts"]).max() <= 0.005 * F
+        check_close(yh[cu_full[b]:cu_full[b + 1]], parts["y"], "bf16", "full window layer")
