@@ -1,0 +1,375 @@
+#!/usr/bin/env python
+"""Benchmark of the Seer hot path on GB300 (prints ONE JSON line on rank 0).
+
+A step is one pass of the whole hot path over one batch of synthetic input:
+step-0 boundary detection (SwiGLU GEMM + fused sparsity count + SNR scan),
+routing + device-resident compaction, and one truncated denoising layer
+(RMSNorm, QKV, varlen bidirectional attention, O projection, SwiGLU MLP).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 2] [--impl ours|reference]
+
+``value``  valid tokens per second of the device-resident step (inputs in HBM);
+``e2e``    the same metric with the host->device copy of the step's input and
+           the device->host copy of its output inside the timed region;
+``--impl reference`` times the CPU oracle on a bounded sample of the same
+workload (the reference arm of this build is the oracle).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "truncated denoise-layer tokens/s & TFLOP/s vs BF16 peak; speedup over padded"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KERNELS_PER_STEP = 11   # detect GEMM, scan, pack, norm, QKV, attn schedule, attn, O proj, norm, gate/up, down
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", type=int, default=2, choices=[0, 1, 2, 4])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def layer_flops(seg, kv, d, F):
+    """Algorithmic FLOPs of one layer (Eq. 2 made exact): projections 8*T*d^2,
+    MLP 6*T*d*F, attention 4*d*sum(L_q * L_kv)."""
+    seg = np.asarray(seg, dtype=np.float64)
+    kv = np.asarray(kv, dtype=np.float64)
+    return float(8.0 * seg.sum() * d * d + 6.0 * seg.sum() * d * F + 4.0 * d * np.sum(seg * kv))
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or self.path is None:
+            return None
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 8:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[4:8]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------------- oracle arm
+_ORACLE_INPUTS = {}
+
+
+def oracle_sample(wl):
+    """Time the CPU oracle on one sequence of the workload (the shortest one):
+    its detection window, boundary scan, and one truncated layer."""
+    import oracle
+    if wl.index not in _ORACLE_INPUTS:
+        lens = synth.lengths(wl)
+        x, cu_full, resp = synth.hidden_full(wl, lens)
+        _ORACLE_INPUTS[wl.index] = (lens, x, cu_full, resp, synth.layer_weights(wl, 0))
+    lens, x, cu_full, resp, w = _ORACLE_INPUTS[wl.index]
+    b = int(np.argmin(lens.full))
+    t0 = time.perf_counter()
+    rows = x[resp[b]:resp[b] + wl.window]
+    counts = oracle.sparsity_counts(rows, w["wg"], w["wu"], wl.act_eps)
+    _, L = oracle.snr_boundary(counts, wl.d_ff)
+    keep = int(lens.ctx[b] + L)
+    seg = x[cu_full[b]:cu_full[b] + keep]
+    oracle.layer_forward_segment(seg, w, wl.n_heads)
+    dt = time.perf_counter() - t0
+    return keep, dt, f"sequence {b} ({keep} kept rows of {int(lens.full[b])}): detection over its {wl.window}-token " \
+                      f"window + one truncated layer, fp64 numpy"
+
+
+def run_reference(args, wl, rank, world):
+    if rank != 0:
+        return
+    cores = len(os.sched_getaffinity(0))
+    for _ in range(args.warmup):
+        oracle_sample(wl)
+    toks, secs = 0, 0.0
+    sample = ""
+    for _ in range(args.steps):
+        k, dt, sample = oracle_sample(wl)
+        toks += k
+        secs += dt
+    v = toks / secs
+    line = {"metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.name, "index": wl.index},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------- our arm
+def main():
+    args = parse()
+    wl = synth.workload(args.workload)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, wl, rank, world)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_14557_gb300 import driver as D
+    from paper_2607_14557_gb300 import seer as S
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(v):
+        if world == 1:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum_over_ranks(v):
+        if world == 1:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        return float(t.item())
+
+    # ---- synthetic inputs, resident in HBM before timing
+    lens = synth.lengths(wl)
+    x_np, cu_full_np, resp_np = synth.hidden_full(wl, lens)
+    w_np = synth.layer_weights(wl, 0)
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    x_host = torch.from_numpy(x_np).to(tdt).pin_memory()
+    x_full = x_host.to(dev)
+    i32 = lambda a: torch.as_tensor(np.asarray(a, dtype=np.int32)).to(dev)
+    cu_full, resp, ctx = i32(cu_full_np), i32(resp_np), i32(lens.ctx)
+    W = D.LayerWeights.from_host(w_np, wl.dtype, dev)
+    W.drop_model_copy()
+    dims = S.make_dims(wl.d, wl.n_heads, wl.head_dim, wl.d_ff)
+    params = S.make_params(wl.act_eps)
+    T_full = int(cu_full_np[-1])
+    path = D.SeerPath(dims, wl.dtype, wl.batch, wl.window, T_full, params, dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        path.step(x_full, cu_full, resp, ctx, W, stream)
+        return path.route()
+
+    # ---- warm-up and the route of this batch
+    for _ in range(max(args.warmup, 3)):
+        route = step()
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == 0
+    L = path.L_star.cpu().numpy()
+    seg = np.diff(path.cu.cpu().numpy())
+    kv = path.kv.cpu().numpy()
+    T_exec = int(seg.sum())
+    T_valid = int(kv.sum())
+    d, F = wl.d, wl.d_ff
+    flops_exec = layer_flops(seg, kv, d, F)
+    flops_valid = layer_flops(kv, kv, d, F)
+    flops_pad = layer_flops(lens.full, lens.full, d, F)
+
+    # ---- timed region: K whole steps (device-resident inputs > L2)
+    barrier()
+    S.seer_profile_reset()
+    S.seer_profile_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        barrier()
+    S.seer_profile_enable(False)
+    ms_step = e0.elapsed_time(e1) / args.steps
+    phases = S.seer_profile_read()
+    ms_step_max = max_over_ranks(ms_step)
+    tokens_all = sum_over_ranks(T_valid)
+    value = tokens_all / (ms_step_max * 1e-3)
+
+    # ---- layer-only timings: truncated vs untruncated (padded) window
+    y_full = torch.empty((T_full, d), dtype=tdt, device=dev)
+
+    def timed(fn, n):
+        for _ in range(2):
+            fn()
+        barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n):
+            fn()
+        b.record(stream)
+        barrier()
+        return a.elapsed_time(b) / n
+
+    ms_layer = timed(lambda: path.layer(W, stream=stream), args.steps)
+    ms_pad = timed(lambda: path.padded_forward(x_full, cu_full, W, y_full, stream), args.steps)
+
+    # ---- end to end through the API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        y_host = torch.empty((T_full, d), dtype=tdt).pin_memory()
+        L_host = torch.empty(wl.batch, dtype=torch.int32).pin_memory()
+
+        def e2e_step():
+            x_full.copy_(x_host, non_blocking=True)
+            r = step()
+            y_host[:r["total"]].copy_(path.y[:r["total"]], non_blocking=True)
+            L_host.copy_(path.L_star, non_blocking=True)
+            return r
+
+        for _ in range(2):
+            e2e_step()
+        barrier()
+        t0 = time.perf_counter()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            r = e2e_step()
+        b.record(stream)
+        barrier()
+        ms_e2e = max_over_ranks(max(a.elapsed_time(b), (time.perf_counter() - t0) * 1e3) / args.steps)
+        h2d = x_host.numel() * x_host.element_size()
+        d2h = r["total"] * d * x_host.element_size() + wl.batch * 4
+        e2e = {"value": tokens_all / (ms_e2e * 1e-3), "unit": "tokens/s", "ms_per_step": ms_e2e,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    assert S.seer_check_device() == 0
+
+    # ---- roofline of the dominant kernel (gate/up GEMM, tensor bound)
+    pk, src = peaks()
+    kernels = {}
+    for name, (ms, n) in phases.items():
+        if n:
+            kernels[name] = {"ms_per_launch": ms / n, "launches": n}
+    flops_of = {"qkv": 6.0 * T_exec * d * d, "o_proj": 2.0 * T_exec * d * d, "gate_up": 4.0 * T_exec * d * F,
+                "down": 2.0 * T_exec * d * F, "attention": 4.0 * d * float(np.sum(seg * kv)),
+                "detect_gemm": 4.0 * wl.batch * wl.window * d * F}
+    for name, fl in flops_of.items():
+        if name in kernels:
+            kernels[name]["tflops"] = fl / (kernels[name]["ms_per_launch"] * 1e-3) / 1e12
+    es = 2 if wl.dtype == "bf16" else 4
+    bytes_of = {"pack": 2.0 * T_exec * d * es, "norm1": T_exec * d * (es + 2), "norm2": T_exec * d * 4}
+    for name, by in bytes_of.items():
+        if name in kernels:
+            kernels[name]["gbs"] = by / (kernels[name]["ms_per_launch"] * 1e-3) / 1e9
+    gu = kernels.get("gate_up", {})
+    achieved = gu.get("tflops")
+    peak = pk["bf16_tflops_sustained"]
+    roofline = {"kernel": "tc_gemm_kernel<Swiglu> (gate/up + SwiGLU)", "bound": "tensor", "achieved": achieved,
+                "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak if achieved else None, "traffic": None,
+                "peak_source": f"{src} bf16 dense, sustained (f16 operands run at the bf16 rate)",
+                "flops_per_launch": flops_of["gate_up"]}
+
+    clocks = clk.summary()
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step_max, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 in/out, f16 tensor-core operands, f32 accumulate" if wl.dtype == "bf16" else "f32",
+        "data": "synthetic",
+        "config": {"workload": f"{wl.name} (workload {wl.index}): batch {wl.batch}, window {wl.window}, "
+                               f"d {wl.d}, heads {wl.n_heads}x{wl.head_dim}, F {wl.d_ff}",
+                   "batch": wl.batch, "window": wl.window, "tokens_full": T_full, "tokens_valid": T_valid,
+                   "tokens_executed": T_exec, "L_star": L.tolist(),
+                   "l2": "inputs larger than L2 (x_full %.0f MB, weights %.0f MB)" % (
+                       T_full * d * es / 1e6, (4 * d * d + 3 * d * F) * 2 / 1e6),
+                   "route": {"groups": route["groups"], "pad_rows": route["pad_rows"], "capacity": route["capacity"]},
+                   "parallelism": f"replicas x{world}"},
+        "layer": {"ms_truncated": ms_layer, "ms_padded": ms_pad, "tflops": flops_exec / (ms_layer * 1e-3) / 1e12,
+                  "frac_of_burst_peak": flops_exec / (ms_layer * 1e-3) / 1e12 / pk["bf16_tflops"],
+                  "frac_of_sustained_peak": flops_exec / (ms_layer * 1e-3) / 1e12 / pk["bf16_tflops_sustained"],
+                  "speedup_vs_padded": ms_pad / ms_layer, "ideal_ratio": flops_pad / flops_valid,
+                  "flops_executed": flops_exec, "flops_valid": flops_valid, "flops_padded": flops_pad},
+        "speedup_step_vs_padded_layer": ms_pad / ms_step,
+        "kernels": kernels, "roofline": roofline, "gpu_launches": KERNELS_PER_STEP * args.steps,
+        "e2e": e2e, "clocks": clocks,
+    }
+    if world == 1 and rank == 0 and not args.no_cpu_baseline:
+        k, dt, sample = oracle_sample(wl)
+        line["cpu_baseline"] = {"value": k / dt, "unit": "tokens/s", "cores": len(os.sched_getaffinity(0)),
+                                "kind": "oracle", "sample": sample, "seconds": dt}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
