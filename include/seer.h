@@ -228,6 +228,23 @@ seer_status seer_swiglu(const void* a, const void* w_gate, const void* w_up, see
                         int B, const int32_t* count_resp_start, int N, float act_eps, int32_t* counts_out,
                         void* stream);
 
+/* seer_attention for callers that cannot allocate device memory, such as code
+ * whose device memory is owned by another allocator (an engine's pool, a
+ * plugin without cudaMalloc) or that must not allocate on its hot path.  The
+ * paper has no counterpart; this is a service of the library.
+ * Same arguments and results as seer_attention, minus the workspace: the
+ * schedule lives in a fixed 1 MiB __device__ array compiled into libseer,
+ * held by every GPU that loads the library until the process exits.
+ * n_heads * (ceil(T_capacity/128) + B) must stay <= 65504, else the call
+ * returns SEER_ERR_WORKSPACE.  The first call on a device looks up the
+ * array's device address (cudaGetSymbolAddress) with that device current,
+ * so make it before any stream capture.  Allocates nothing.  Every call
+ * reuses the same array: calls whose kernels overlap on the GPU race and must
+ * not be issued (nothing in the array needs to start at zero). */
+seer_status seer_attention_noalloc(const void* qkv, void* o, seer_dtype dt, const int32_t* cu_seqlens,
+                                   const int32_t* kv_len, int B, int T_capacity, int n_heads, int head_dim,
+                                   void* stream);
+
 /* dst[i] = src[i] converted (round to nearest even) for i < n; n % 8 == 0.
  * bf16 -> f16 is exact for |v| >= 2^-14 and below 65504 (f16's normal range).
  * Used once per model to make the f16 weight copies of bf16 layers. */

@@ -16,7 +16,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libseer.so")
-SOURCES = ["seer_api.cu", "tc_gemm.cu", "tc_attn.cu", "simt.cu", "aux_kernels.cu"]
+SOURCES = ["seer_api.cu", "tc_gemm.cu", "tc_attn.cu", "simt.cu", "aux_kernels.cu", "seer_noalloc.cu"]
 HEADERS = ["common.cuh", "kernels.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -77,6 +77,9 @@ cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_
                               int eager_max_bucket, void* x_packed, int* cu_out, int* kv_out, int* meta_out,
                               int* host_ctrl_dev, int epoch, int* err, int num_sms, cudaStream_t st);
 
+// Sets the message returned by seer_last_error() on this thread.
+void set_last_error(const char* msg);
+
 constexpr int kCtrlMaxGroups = 32;
 constexpr int kCtrlWords = 8 + 4 * kCtrlMaxGroups;
 

@@ -371,6 +371,12 @@ seer_status do_attention(const void* qkv, void* o, seer_dtype dt, const int32_t*
 
 }  // namespace
 
+namespace seer {
+// Lets other translation units of the library report a message through
+// seer_last_error().
+void set_last_error(const char* msg) { g_msg = msg; }
+}  // namespace seer
+
 extern "C" {
 
 const char* seer_last_error(void) { return g_msg.c_str(); }

@@ -1,0 +1,84 @@
+// seer_attention_noalloc: the varlen attention entry point for callers that
+// must not allocate device memory.
+//
+// seer_attention needs a small scratch buffer for its work schedule, which the
+// caller normally passes in.  Some callers cannot provide one: code that runs
+// where the device memory is entirely owned by another allocator (a serving
+// engine's memory pool, a plugin with no access to cudaMalloc), or that must
+// not allocate at all on its hot path.  For them this entry point uses a
+// fixed scratch array compiled into the library instead.
+//
+// The array is a file-scope __device__ variable of kScratchBytes (1 MiB), so
+// every GPU that loads libseer holds it until the process exits.  Host code
+// only sees a host-side stand-in for it; the device address is looked up once
+// per device with cudaGetSymbolAddress on the first call made while that
+// device is current.  That first call therefore performs set-up and should
+// come before any CUDA stream capture.  No call allocates or frees memory.
+//
+// All calls share the one array and leave their schedule in it.  Nothing in
+// it has to start at zero: the schedule kernel rewrites the entries and the
+// count it uses on every call.  Calls whose kernels overlap on the GPU (for
+// example on two streams at once) race on the array and must not be issued.
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <mutex>
+
+#include "../../include/seer.h"
+#include "kernels.h"
+
+namespace {
+
+constexpr size_t kScratchBytes = size_t(1) << 20;
+
+static __device__ __align__(256) unsigned char g_attn_scratch[kScratchBytes];
+
+std::mutex g_mu;
+void* g_scratch_addr[64] = {};
+
+// Bytes of schedule the attention kernels use: H * (ceil(T/128) + B) int4
+// entries rounded up to 256 bytes, plus 256 bytes for the entry count.
+size_t schedule_bytes(int T_cap, int B, int H) {
+  const size_t units = static_cast<size_t>(H) * (static_cast<size_t>((T_cap + 127) / 128) + static_cast<size_t>(B));
+  return ((units * 16 + 255) & ~size_t(255)) + 256;
+}
+
+}  // namespace
+
+extern "C" seer_status seer_attention_noalloc(const void* qkv, void* o, seer_dtype dt, const int32_t* cu_seqlens,
+                                              const int32_t* kv_len, int B, int T_capacity, int n_heads, int head_dim,
+                                              void* stream) {
+  if (B <= 0 || T_capacity < 0 || n_heads <= 0) {
+    seer::set_last_error("seer_attention_noalloc: bad sizes");
+    return SEER_ERR_INVALID_ARG;
+  }
+  const size_t need = schedule_bytes(T_capacity, B, n_heads);
+  if (need > kScratchBytes) {
+    seer::set_last_error("seer_attention_noalloc: this batch needs a larger schedule than the built-in scratch "
+                         "of 1 MiB holds (n_heads * (ceil(T_capacity/128) + B) must stay <= 65504); use "
+                         "seer_attention with a caller-provided workspace");
+    return SEER_ERR_WORKSPACE;
+  }
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= 64) {
+    seer::set_last_error("seer_attention_noalloc: no usable current device");
+    return SEER_ERR_CUDA;
+  }
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (g_scratch_addr[dev] == nullptr) {
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_attn_scratch);
+      if (e != cudaSuccess) {
+        seer::set_last_error("seer_attention_noalloc: cudaGetSymbolAddress of the scratch array failed");
+        return SEER_ERR_CUDA;
+      }
+      g_scratch_addr[dev] = p;
+    }
+    scratch = g_scratch_addr[dev];
+  }
+  return seer_attention(qkv, o, dt, cu_seqlens, kv_len, B, T_capacity, n_heads, head_dim, scratch, kScratchBytes,
+                        stream);
+}

@@ -78,6 +78,7 @@ def lib() -> ctypes.CDLL:
             "seer_swiglu": [vp, vp, vp, i32, vp, i32, i32, vp, i32, i32, vp, i32, vp, i32, ctypes.c_float, vp, vp],
             "seer_convert": [vp, i32, vp, i32, sz, vp],
             "seer_attention": [vp, vp, i32, vp, vp, i32, i32, i32, i32, vp, sz, vp],
+            "seer_attention_noalloc": [vp, vp, i32, vp, vp, i32, i32, i32, i32, vp],
             "seer_check_device": [ctypes.POINTER(ctypes.c_int)],
             "seer_profile_enable": [i32],
             "seer_profile_reset": [],
@@ -200,6 +201,11 @@ def seer_attention(qkv, o, dt, cu_seqlens, kv_len, B, T_capacity, n_heads, head_
                    stream=None):
     _check(lib().seer_attention(_p(qkv), _p(o), _dt(dt), _p(cu_seqlens), _p(kv_len), B, T_capacity, n_heads,
                                 head_dim, _p(ws), ws_bytes, _stream(stream)))
+
+
+def seer_attention_noalloc(qkv, o, dt, cu_seqlens, kv_len, B, T_capacity, n_heads, head_dim, stream=None):
+    _check(lib().seer_attention_noalloc(_p(qkv), _p(o), _dt(dt), _p(cu_seqlens), _p(kv_len), B, T_capacity, n_heads,
+                                        head_dim, _stream(stream)))
 
 
 def seer_check_device() -> int:
