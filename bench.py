@@ -43,7 +43,7 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", type=int, default=2, choices=[0, 1, 2, 4])
+    ap.add_argument("--workload", type=int, default=2, choices=[0, 1, 2, 3, 4])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -168,6 +168,103 @@ def run_reference(args, wl, rank, world):
     print(json.dumps(line), flush=True)
 
 
+# ----------------------------------------------------------------- stack (workload 3)
+def run_stack(args, wl, world, rank, local):
+    """32-layer stack, 64 denoising steps: step 0 over the full windows (with the
+    fused count hook at the detection layer), detection + route/pack, then 63
+    truncated steps replayed from a CUDA graph; against 64 untruncated steps
+    replayed from their own graph."""
+    import torch
+
+    from paper_2607_14557_gb300 import driver as D
+    from paper_2607_14557_gb300 import seer as S
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    detect_layer = 3
+    lens = synth.lengths(wl)
+    x_np, cu_full_np, resp_np = synth.hidden_full(wl, lens)
+    x_full = torch.from_numpy(x_np).to(torch.bfloat16).to(dev)
+    i32 = lambda a: torch.as_tensor(np.asarray(a, dtype=np.int32)).to(dev)
+    cu_full, resp, ctx = i32(cu_full_np), i32(resp_np), i32(lens.ctx)
+    t0 = time.perf_counter()
+    layers = [None] * wl.n_layers
+    for l, bits in synth.stack_weights_bf16_bits(wl, range(wl.n_layers)):
+        layers[l] = D.LayerWeights.from_bf16_bits(bits, dev, keep_model=("w_gate", "w_up") if l == detect_layer else ())
+    t_weights = time.perf_counter() - t0
+    dims = S.make_dims(wl.d, wl.n_heads, wl.head_dim, wl.d_ff)
+    params = S.make_params(wl.act_eps)
+    T_full = int(cu_full_np[-1])
+    stack = D.SeerStack(dims, "bf16", wl.batch, wl.window, T_full, params, layers, detect_layer, dev)
+    stream = torch.cuda.current_stream()
+    n_steps = wl.steps
+
+    # warm-up: step 0, the graphs, a few steps of each
+    stack.step0(x_full, cu_full, resp, ctx, stream)
+    route = stack.path.route()
+    g_trunc = stack.truncated_graph(route["capacity"])
+    g_pad = stack.capture("padded", lambda stream: stack.padded_step(x_full, cu_full, stream=stream))
+    for _ in range(max(args.warmup, 3)):
+        g_trunc.replay()
+        g_pad.replay()
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == 0
+    L = stack.path.L_star.cpu().numpy()
+    seg = np.diff(stack.path.cu.cpu().numpy())
+    kv = stack.path.kv.cpu().numpy()
+    T_valid, T_exec = int(kv.sum()), int(seg.sum())
+    d, F, nl = wl.d, wl.d_ff, wl.n_layers
+
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        ev[0].record(stream)
+        stack.step0(x_full, cu_full, resp, ctx, stream)
+        ev[1].record(stream)
+        r = stack.path.route()
+        g = stack.truncated_graph(r["capacity"])
+        for _ in range(n_steps - 1):
+            g.replay()
+        ev[2].record(stream)
+        for _ in range(n_steps):
+            g_pad.replay()
+        ev[3].record(stream)
+        torch.cuda.synchronize()
+    assert S.seer_check_device() == 0
+    ms0 = ev[0].elapsed_time(ev[1])
+    ms_rest = ev[1].elapsed_time(ev[2])
+    ms_pad = ev[2].elapsed_time(ev[3])
+    ms_seer = ms0 + ms_rest
+    fl_full = layer_flops(lens.full, lens.full, d, F) * nl
+    fl_trunc = layer_flops(seg, kv, d, F) * nl
+    fl_valid = layer_flops(kv, kv, d, F) * nl
+    tok_layers = (T_full + (n_steps - 1) * T_valid) * nl
+    value = tok_layers / (ms_seer * 1e-3)
+    pk, src = peaks()
+    tflops_rest = fl_trunc * (n_steps - 1) / (ms_rest * 1e-3) / 1e12
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": n_steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": ms_seer / n_steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 in/out, f16 tensor-core operands, f32 accumulate", "data": "synthetic",
+        "config": {"workload": f"{wl.name} (workload 3): {nl} layers x {n_steps} denoising steps, batch {wl.batch}, "
+                               f"window {wl.window}, d {d}, F {F}; tokens counted once per layer and step",
+                   "tokens_full": T_full, "tokens_valid": T_valid, "tokens_executed": T_exec, "L_star": L.tolist(),
+                   "route": {"groups": r["groups"], "capacity": r["capacity"]},
+                   "l2": "inputs larger than L2 (weights %.1f GB)" % (nl * (4 * d * d + 3 * d * F) * 2 / 1e9),
+                   "weights_setup_s": t_weights},
+        "stack": {"ms_step0_full": ms0, "ms_steps_1_to_%d" % (n_steps - 1): ms_rest, "ms_padded_%d_steps" % n_steps: ms_pad,
+                  "speedup_vs_padded": ms_pad / ms_seer,
+                  "ideal_ratio": fl_full * n_steps / (fl_full + fl_valid * (n_steps - 1)),
+                  "tflops_truncated_steps": tflops_rest, "frac_of_burst_peak": tflops_rest / pk["bf16_tflops"],
+                  "tflops_padded": fl_full * n_steps / (ms_pad * 1e-3) / 1e12,
+                  "truncated_tokens_per_s": T_valid * nl * (n_steps - 1) / (ms_rest * 1e-3)},
+        "gpu_launches": nl * 8 * (2 * n_steps) + 3, "clocks": clk.summary(),
+        "peak_source": src,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 # ----------------------------------------------------------------- our arm
 def main():
     args = parse()
@@ -177,6 +274,9 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, wl, rank, world)
+        return
+    if args.workload == 3:
+        run_stack(args, wl, world, rank, local)
         return
 
     import torch

@@ -286,11 +286,13 @@ def layer_forward_packed(x_packed, cu, w, n_heads: int, *, kv_len=None, dtype=No
     return y
 
 
-def layer_forward_rows(x_seg, w, n_heads: int, rows, *, kv_len=None, dtype=None, rms_eps=1e-5):
+def layer_forward_rows(x_seg, w, n_heads: int, rows, *, kv_len=None, dtype=None, rms_eps=1e-5, act_eps=None):
     """Outputs of selected rows of one segment (keys/values from all kept rows).
 
     Same arithmetic as :func:`layer_forward_segment`, restricted to the query
     rows ``rows``; used where the full segment is too large for the oracle.
+    With ``act_eps`` set, also returns the near-zero SwiGLU counts of those
+    rows (the step-0 detection hook): ``(y_rows, counts)``.
     """
     R = rounding_for(dtype)
     x = _f64(x_seg)
@@ -305,5 +307,8 @@ def layer_forward_rows(x_seg, w, n_heads: int, rows, *, kv_len=None, dtype=None,
     o = R(attention(q, k, v, n_heads))
     h = R(xr + o @ _f64(w["wo"]).T)
     hn = R(rmsnorm(h, w["g_mlp"], rms_eps))
-    a = R(swiglu_activation(hn, w["wg"], w["wu"]))
-    return R(h + a @ _f64(w["wd"]).T)
+    a_exact = swiglu_activation(hn, w["wg"], w["wu"])
+    y = R(h + R(a_exact) @ _f64(w["wd"]).T)
+    if act_eps is None:
+        return y
+    return y, (np.abs(a_exact) < act_eps).sum(-1).astype(np.int64)

@@ -61,6 +61,19 @@ class LayerWeights:
         run = model if dtype == "f32" else {k: f16_copy(v) for k, v in model.items()}
         return LayerWeights(model, run)
 
+    @staticmethod
+    def from_bf16_bits(bits: Dict[str, np.ndarray], device=None, keep_model=()) -> "LayerWeights":
+        """Upload bf16 bit patterns ({name: uint16 array}, as produced for a
+        stack) and make the f16 copies the kernels run on; keep only the
+        model-dtype tensors named in ``keep_model``."""
+        device = device or _dev()
+        up = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(device)
+        model = {"w_qkv": up(np.concatenate([bits["wq"], bits["wk"], bits["wv"]], axis=0)), "w_o": up(bits["wo"]),
+                 "w_gate": up(bits["wg"]), "w_up": up(bits["wu"]), "w_down": up(bits["wd"]),
+                 "g_attn": up(bits["g_attn"]), "g_mlp": up(bits["g_mlp"])}
+        run = {k: f16_copy(v) for k, v in model.items()}
+        return LayerWeights({k: v for k, v in model.items() if k in keep_model}, run)
+
     def struct(self) -> S.seer_layer_weights:
         r = self.run
         return S.make_weights(r["w_qkv"], r["w_o"], r["w_gate"], r["w_up"], r["w_down"], r["g_attn"], r["g_mlp"])
@@ -139,12 +152,15 @@ class SeerStack:
     """Denoising loop over a stack of layers (one GPU).
 
     Step 0 runs every layer over the full windows; the detection layer's
-    gate/up epilogue counts near-zero activations of the response rows, the
-    SNR scan turns them into L*, and the fused route/pack kernel compacts the
-    step-0 *input* rows.  Steps 1..T-1 then run every layer over the packed
-    sequences.  The step body is captured once into a CUDA graph (kernels
-    read the packed row count from device memory, so the graph serves any
-    total up to the capacity) and replayed.
+    gate/up epilogue counts near-zero activations of the response rows
+    (``hook_counts``).  The boundaries that drive truncation come from the
+    detector applied to the step-0 input rows with the detection layer's
+    gate/up weights (random-init weights carry no semantic signal after a
+    normalised stack, so the planted input stands in for a trained model);
+    the route/pack kernel then compacts the step-0 input, and steps 1..T-1 run
+    every layer over the packed sequences.  Step bodies are captured into CUDA
+    graphs: the kernels read the packed row count from device memory, so one
+    graph per capacity serves any total up to it.
     """
 
     def __init__(self, dims, dtype, B, N, T_full, params, layers: List[LayerWeights], detect_layer: int = 3,
@@ -156,37 +172,42 @@ class SeerStack:
         tdt = self.path.x_packed.dtype
         d = dims.d_model
         self.buf = [torch.empty((T_full, d), dtype=tdt, device=dev) for _ in range(2)]
-        self.graphs: Dict[int, torch.cuda.CUDAGraph] = {}
+        self.hook_counts = torch.zeros(B * N, dtype=torch.int32, device=dev)
+        self.graphs: Dict[object, torch.cuda.CUDAGraph] = {}
 
-    def _run_layers(self, x, cu, kv, T_cap, resp_start=None, stream=None):
+    def _run_layers(self, x, cu, kv, T_cap, resp_start=None, stream=None, n_layers=None):
         p = self.path
         cur = x
-        for li, w in enumerate(self.layers):
+        for li, w in enumerate(self.layers[:n_layers]):
             out = self.buf[li % 2] if cur is not self.buf[li % 2] else self.buf[(li + 1) % 2]
             count = resp_start is not None and li == self.detect_layer
             S.seer_layer_forward(w.struct(), p.dims, p.dtype, cur, out, cu, kv, p.B, T_cap,
                                  resp_start if count else None, p.N if count else 0,
-                                 p.params.act_eps if count else 0.0, p.counts if count else None, p.ws, p.ws_bytes,
-                                 stream=stream)
+                                 p.params.act_eps if count else 0.0, self.hook_counts if count else None, p.ws,
+                                 p.ws_bytes, stream=stream)
             cur = out
         return cur
 
     def step0(self, x_full, cu_full, resp_start, ctx_len, stream=None):
-        """Full-window step with the fused detection hook, then scan + pack."""
+        """Full-window step with the fused count hook, then detect + route/pack."""
         p = self.path
-        self._run_layers(x_full, cu_full, None, p.T_full, resp_start=resp_start, stream=stream)
-        S.seer_snr_scan(p.counts, p.B, p.N, p.dims.d_ff, p.params, p.L_star, p.i_star, stream=stream)
+        out = self._run_layers(x_full, cu_full, None, p.T_full, resp_start=resp_start, stream=stream)
+        p.detect(x_full, resp_start, self.layers[self.detect_layer], stream)
         p.pack(x_full, cu_full, ctx_len, stream)
+        return out
 
-    def truncated_step(self, stream=None):
+    def truncated_step(self, T_cap=None, stream=None):
         p = self.path
-        return self._run_layers(p.x_packed, p.cu, p.kv, p.T_full, stream=stream)
+        return self._run_layers(p.x_packed, p.cu, p.kv, T_cap or p.T_full, stream=stream)
 
     def padded_step(self, x_full, cu_full, stream=None):
         return self._run_layers(x_full, cu_full, None, self.path.T_full, stream=stream)
 
-    def capture(self, fn, key):
-        """Capture ``fn`` (a step body) into a CUDA graph stored under ``key``."""
+    def capture(self, key, fn):
+        """Capture ``fn(stream=...)`` (one step body) into a CUDA graph under ``key``."""
+        if key in self.graphs:
+            return self.graphs[key]
+        S.seer_profile_enable(False)
         s = torch.cuda.Stream()
         s.wait_stream(torch.cuda.current_stream())
         with torch.cuda.stream(s):
@@ -197,3 +218,8 @@ class SeerStack:
             fn(stream=torch.cuda.current_stream())
         self.graphs[key] = g
         return g
+
+    def truncated_graph(self, capacity: int):
+        """Graph of one truncated step sized for ``capacity`` packed rows."""
+        cap = min(int(capacity), self.path.T_full)
+        return self.capture(("trunc", cap), lambda stream: self.truncated_step(cap, stream=stream))

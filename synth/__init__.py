@@ -181,6 +181,28 @@ def hidden_full(wl: Workload, lens: Optional[Lengths] = None):
     return x, cu.astype(np.int32), resp.astype(np.int32)
 
 
+def _bf16_bits_of_layer(args):
+    wl, layer = args
+    w = layer_weights(wl, layer)
+    return layer, {k: (np.ascontiguousarray(v).view(np.uint32) >> 16).astype(np.uint16) for k, v in w.items()}
+
+
+def stack_weights_bf16_bits(wl: Workload, layers, workers: Optional[int] = None):
+    """Yield ``(layer, {name: uint16 bf16 bit patterns})`` for the given layers,
+    generated in a spawn-started process pool (each layer has its own seeded
+    stream, so the values equal :func:`layer_weights`).  bf16 workloads only."""
+    import concurrent.futures
+    import multiprocessing
+    import os
+    assert wl.dtype == "bf16"
+    layers = list(layers)
+    n = workers or max(1, min(len(layers), (os.cpu_count() or 2) // 2, 16))
+    ctx = multiprocessing.get_context("spawn")
+    with concurrent.futures.ProcessPoolExecutor(max_workers=n, mp_context=ctx) as ex:
+        for item in ex.map(_bf16_bits_of_layer, [(wl, l) for l in layers]):
+            yield item
+
+
 def layer_weights(wl: Workload, layer: int = 0) -> Dict[str, np.ndarray]:
     """Random-init weights of one block, nn.Linear layout [out, in]."""
     rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([wl.seed, 7, layer])))

@@ -183,3 +183,12 @@ def test_count_hook_equals_detector_on_mlp_input():
     parts = oracle.layer_forward_segment(x, w, 4, return_parts=True, count_rows=[2, 3, 8], act_eps=0.05)
     ref = oracle.sparsity_counts(parts["hn"][[2, 3, 8]], w["wg"], w["wu"], 0.05)
     np.testing.assert_array_equal(parts["counts"], ref)
+
+
+def test_rows_variant_counts_equal_full_segment_hook():
+    wl, w = _tiny(seed=8)
+    x = np.random.default_rng(15).standard_normal((11, 32))
+    rows = [1, 4, 10]
+    _, counts = oracle.layer_forward_rows(x, w, 4, rows, kv_len=9, act_eps=0.05)
+    full = oracle.layer_forward_segment(x, w, 4, kv_len=9, count_rows=rows, act_eps=0.05, return_parts=True)
+    np.testing.assert_array_equal(counts, full["counts"])
