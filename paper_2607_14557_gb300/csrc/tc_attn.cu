@@ -5,17 +5,21 @@
 // the first kv_len[b] rows of the same segment, with no causal mask; rows
 // beyond kv_len (bucket padding of the static path) are never keys.
 //
-// One CTA per (segment, head, 128-query tile); 192 threads:
+// One CTA per (segment, head, 128-query tile); 64 + 128 * NGRP threads:
 //   warp 0     TMA producer: Q tile once, then K_j and V_j (128 keys x 128
 //              dims, 128-byte swizzle) into a 2-deep ring;
 //   warp 1     TMEM allocator + MMA issuer: S_j = Q K_j^T (M=N=128, K=16 x 8)
 //              into one of two S buffers, then O += P_j V_j (V as an MN-major
 //              operand) into the O accumulator;
-//   warps 2-5  softmax: each thread owns one query row (one TMEM lane),
-//              online softmax in the log2 domain with lazy rescaling (O is
-//              only rescaled in TMEM when the running max grows by more than
-//              2^8), P_j written to shared memory in the swizzled K-major
-//              layout the tensor core reads, final O / l epilogue.
+//   warps 2.. softmax, NGRP groups of four warps: a query row (one TMEM
+//              lane) is shared by one thread of each group, which owns
+//              128 / NGRP of the key columns (and of the output dims); the
+//              parts of a row exchange their maxima through shared memory
+//              once per key tile (an mbarrier, so every wait is bounded).
+//              Online softmax in the log2 domain with lazy rescaling: O is
+//              rescaled in TMEM only when the running max grows by more than
+//              2^8.  P_j goes to shared memory in the swizzled K-major layout
+//              the tensor core reads.
 // The QK^T MMA of tile j+1 overlaps the softmax of tile j.
 // The schedule kernel orders work units longest segment first.
 #include <math.h>
@@ -29,17 +33,27 @@ namespace {
 constexpr int BQ = 128;
 constexpr int BKV = 128;
 constexpr int DH = 128;
-constexpr int THREADS = 192;
-constexpr int TILE_BYTES = 128 * DH * 2;   // 32 KB: 128 rows x 128 bf16 as two 16 KB swizzle panels
+constexpr int NGRP = 2;                     // softmax column groups (4 warps each)
+constexpr int COLS = BKV / NGRP;            // key columns / output dims per softmax thread
+constexpr int SOFTMAX_WARPS = 4 * NGRP;
+constexpr int THREADS = 64 + 32 * SOFTMAX_WARPS;
+constexpr int TILE_BYTES = 128 * DH * 2;   // 32 KB: 128 rows x 128 16-bit values as two 16 KB swizzle panels
 constexpr int PANEL = 16384;
 constexpr int OFF_Q = 0;
 constexpr int OFF_K = TILE_BYTES;           // 2 buffers
 constexpr int OFF_V = 3 * TILE_BYTES;       // 2 buffers
 constexpr int OFF_P = 5 * TILE_BYTES;
 constexpr int OFF_BAR = 6 * TILE_BYTES;
-constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+constexpr int OFF_RED = OFF_BAR + 256;      // float max[2 tiles][NGRP][128] + float sum[NGRP][128]
+constexpr int SMEM_BYTES = OFF_RED + (2 * NGRP * 128 + NGRP * 128) * 4 + 1024;
 constexpr uint32_t TMEM_COLS = 512;         // S0 [0,128), S1 [128,256), O [256,384)
 constexpr float RESCALE_THRESHOLD = 8.0f;   // log2 units
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 template <bool F16>
 __global__ void __launch_bounds__(THREADS, 1)
@@ -68,8 +82,12 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint64_t* s_empty = bars + 11;   // [2]
   uint64_t* p_full = bars + 13;
   uint64_t* pv_done = bars + 14;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 15);
+  uint64_t* max_ready = bars + 15; // [2] row-max exchange, one per tile parity
+  uint64_t* sum_ready = bars + 17;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* red_max = reinterpret_cast<float*>(smem + OFF_RED);   // [2 tiles][NGRP][128] partial row maxima
+  float* red_sum = red_max + 2 * NGRP * 128;                   // [NGRP][128] partial row sums
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -82,10 +100,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(&v_full[i], 1);
       mbar_init(&v_empty[i], 1);
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_empty[i], 4);
+      mbar_init(&s_empty[i], SOFTMAX_WARPS);
+      mbar_init(&max_ready[i], SOFTMAX_WARPS);
     }
-    mbar_init(p_full, 4);
+    mbar_init(p_full, SOFTMAX_WARPS);
     mbar_init(pv_done, 1);
+    mbar_init(sum_ready, SOFTMAX_WARPS);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -163,7 +183,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int k = 0; k < DH / 16; ++k) {
           const uint32_t off = (k >> 2) * PANEL + (k & 3) * 32;
           tc_mma_f16(tmem + sb * 128, make_sdesc_sw128(sq + off, 16, 1024), make_sdesc_sw128(sk + off, 16, 1024),
-                      idesc_qk, k > 0 ? 1u : 0u);
+                     idesc_qk, k > 0 ? 1u : 0u);
         }
         tc_commit(&k_empty[sb]);
         tc_commit(&s_full[sb]);
@@ -172,65 +192,95 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (ok && nkv > 0) issue_pv(nkv - 1);
     }
   } else {
-    // -------------------------------------------------- softmax warps 2..5
+    // -------------------------------------------------- softmax warps 2..
+    const int grp = (warp - 2) >> 2;              // column group: keys / output dims [COLS grp, COLS grp + COLS)
     const int qw = warp & 3;
     const int r = qw * 32 + lane;                 // query row inside the tile == TMEM lane
+    const int col0 = grp * COLS;
     const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
     const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
-    uint8_t* sP = smem + OFF_P;
-    float m_ref = -INFINITY;
-    float l = 0.f;
+    // P row r, keys [col0, col0 + COLS): 16-byte chunks (col0 % 64) / 8 + c of
+    // panel col0 / 64 in the swizzled K-major layout (chunk k of row r sits at
+    // (r / 8) * 1024 + (r % 8) * 128 + ((k ^ (r % 8)) * 16))
+    uint8_t* sProw = smem + OFF_P + (col0 / 64) * PANEL + (r >> 3) * 1024 + (r & 7) * 128;
+    const int chunk0 = (col0 % 64) / 8;
+    float m_ref = -INFINITY;                      // running max, log2 units
+    float l = 0.f;                                // partial row sum over this thread's columns
     bool ok = true;
     for (int j = 0; j < nkv; ++j) {
       const int sb = j & 1, use = j >> 1;
       if (!mbar_wait(&s_full[sb], use & 1, abort_flag, p.err)) { ok = false; break; }
       tc_fence_after();
-      float s[BKV];
+      float s[COLS];
+      {
+        uint32_t ra[COLS / 32][32];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t rr[32];
-        tmem_ld32(tmem + lane_off + sb * 128 + c * 32, rr);
+        for (int c = 0; c < COLS / 32; ++c) tmem_ld32(tmem + lane_off + sb * 128 + col0 + 32 * c, ra[c]);
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(rr[i]);
+        for (int c = 0; c < COLS / 32; ++c)
+#pragma unroll
+          for (int i = 0; i < 32; ++i) s[32 * c + i] = __uint_as_float(ra[c][i]);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_empty[sb]);
 
-      const int valid = kvL - j * BKV;            // >= 1
-      float mt = -INFINITY;
+      const int valid_all = kvL - j * BKV;        // keys of this tile, >= 1
+      const int valid = valid_all - col0;         // keys of this group (may be <= 0 or >= COLS)
+      if (valid < COLS) {
 #pragma unroll
-      for (int c = 0; c < BKV; ++c) {
-        const float v = c < valid ? s[c] * scale_log2 : -INFINITY;
-        s[c] = v;
-        mt = fmaxf(mt, v);
+        for (int c = 0; c < COLS; ++c) s[c] = c < valid ? s[c] : -INFINITY;
       }
+      // tree-shaped max over this group's columns, then exchange with the
+      // other groups of the row (double-buffered by tile parity, bounded wait)
+      float mx[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mx[i] = s[i];
+#pragma unroll
+      for (int c = 8; c < COLS; c += 8) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mx[i] = fmaxf(mx[i], s[c + i]);
+      }
+      const float mloc = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      float* rm = red_max + (j & 1) * (NGRP * 128);
+      rm[grp * 128 + r] = mloc;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&max_ready[j & 1]);
+      if (!mbar_wait(&max_ready[j & 1], use & 1, abort_flag, p.err)) { ok = false; break; }
+      float mall = rm[r];
+#pragma unroll
+      for (int g = 1; g < NGRP; ++g) mall = fmaxf(mall, rm[g * 128 + r]);
+      const float mt = mall * scale_log2;
       const float m_new = fmaxf(m_ref, mt);
       const bool need = (j == 0) || (m_new > m_ref + RESCALE_THRESHOLD);
       float alpha = 1.f;
       if (need) {
-        alpha = (j == 0) ? 0.f : exp2f(m_ref - m_new);
+        alpha = (j == 0) ? 0.f : ex2(m_ref - m_new);
         m_ref = m_new;
       }
-      float rs = 0.f;
+      const float neg = -m_ref;
+      float rs[4] = {0.f, 0.f, 0.f, 0.f};
+      uint32_t pk[COLS / 2];
 #pragma unroll
-      for (int c = 0; c < BKV; c += 2) {
-        const uint32_t pk = pack2(exp2f(s[c] - m_ref), exp2f(s[c + 1] - m_ref), F16);
-        rs += lo16(pk, F16) + hi16(pk, F16);
-        s[c] = __uint_as_float(pk);               // keep the packed pair
+      for (int c = 0; c < COLS; c += 2) {
+        const float p0 = ex2(fmaf(s[c], scale_log2, neg));
+        const float p1 = ex2(fmaf(s[c + 1], scale_log2, neg));
+        rs[(c >> 1) & 3] += p0 + p1;
+        pk[c >> 1] = pack2(p0, p1, F16);
       }
-      l = l * alpha + rs;
+      l = l * alpha + ((rs[0] + rs[1]) + (rs[2] + rs[3]));
 
-      if (valid < BKV) {
-        // last, partial key tile: clear the value rows past kv_len so that
-        // stale data (possibly non-finite) cannot meet the zero probabilities
+      if (valid_all < BKV && grp < 2) {
+        // last, partial key tile: groups 0 and 1 clear value panels 0 and 1
+        // of the rows past kv_len so stale (possibly non-finite) data cannot
+        // meet the zero probabilities
         if (!mbar_wait(&v_full[sb], use & 1, abort_flag, p.err)) { ok = false; break; }
-        if (r >= valid) {
-          uint4* v0 = reinterpret_cast<uint4*>(smem + OFF_V + sb * TILE_BYTES + r * 128);
-          uint4* v1 = reinterpret_cast<uint4*>(smem + OFF_V + sb * TILE_BYTES + PANEL + r * 128);
+        if (r >= valid_all) {
+          uint4* v = reinterpret_cast<uint4*>(smem + OFF_V + sb * TILE_BYTES + grp * PANEL + r * 128);
 #pragma unroll
-          for (int i = 0; i < 8; ++i) { v0[i] = make_uint4(0, 0, 0, 0); v1[i] = make_uint4(0, 0, 0, 0); }
+          for (int i = 0; i < 8; ++i) v[i] = make_uint4(0, 0, 0, 0);
         }
       }
       if (j > 0) {
@@ -238,9 +288,9 @@ __global__ void __launch_bounds__(THREADS, 1)
         tc_fence_after();
         if (__any_sync(0xffffffffu, need)) {
 #pragma unroll 1
-          for (int c = 0; c < 4; ++c) {
+          for (int c = 0; c < COLS / 32; ++c) {
             uint32_t rr[32];
-            const uint32_t ta = tmem + lane_off + 256 + c * 32;
+            const uint32_t ta = tmem + lane_off + 256 + col0 + 32 * c;
             tmem_ld32(ta, rr);
             tmem_ld_wait();
 #pragma unroll
@@ -250,34 +300,39 @@ __global__ void __launch_bounds__(THREADS, 1)
           tmem_st_wait();
         }
       }
-      // P row r -> swizzled K-major layout: 16-byte chunk c of row r lives at
-      // panel (c / 8), offset (r / 8) * 1024 + (r % 8) * 128 + ((c % 8) ^ (r % 8)) * 16
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        const int panel = c >> 3;
-        const int chunk = (c & 7) ^ (r & 7);
-        uint4* dst = reinterpret_cast<uint4*>(sP + panel * PANEL + (r >> 3) * 1024 + (r & 7) * 128 + chunk * 16);
-        *dst = make_uint4(__float_as_uint(s[8 * c + 0]), __float_as_uint(s[8 * c + 2]), __float_as_uint(s[8 * c + 4]),
-                          __float_as_uint(s[8 * c + 6]));
+      for (int c = 0; c < COLS / 8; ++c) {
+        uint4* dst = reinterpret_cast<uint4*>(sProw + (((chunk0 + c) ^ (r & 7)) * 16));
+        *dst = make_uint4(pk[4 * c + 0], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
       }
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full);
     }
-    if (ok && nkv > 0 && mbar_wait(pv_done, (nkv - 1) & 1, abort_flag, p.err)) {
+    if (ok && nkv > 0) {
+      red_sum[grp * 128 + r] = l;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sum_ready);
+      ok = mbar_wait(sum_ready, 0, abort_flag, p.err) && mbar_wait(pv_done, (nkv - 1) & 1, abort_flag, p.err);
+    }
+    if (ok && nkv > 0) {
       tc_fence_after();
-      const float inv_l = 1.f / l;
+      float lsum = 0.f;
+#pragma unroll
+      for (int g = 0; g < NGRP; ++g) lsum += red_sum[g * 128 + r];
+      const float inv_l = 1.f / lsum;
       const int row = q0 + r;
       const bool valid_row = (qt * BQ + r) < L;
-      uint16_t* orow = reinterpret_cast<uint16_t*>(p.out) + static_cast<size_t>(valid_row ? row : 0) * p.ldo + h * DH;
+      uint16_t* orow =
+          reinterpret_cast<uint16_t*>(p.out) + static_cast<size_t>(valid_row ? row : 0) * p.ldo + h * DH + col0;
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 0; c < COLS / 32; ++c) {
         uint32_t rr[32];
-        tmem_ld32(tmem + lane_off + 256 + c * 32, rr);
+        tmem_ld32(tmem + lane_off + 256 + col0 + 32 * c, rr);
         tmem_ld_wait();
         if (valid_row) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+          uint4* dst = reinterpret_cast<uint4*>(orow + 32 * c);
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             dst[i] = make_uint4(pack2(__uint_as_float(rr[8 * i + 0]) * inv_l, __uint_as_float(rr[8 * i + 1]) * inv_l, F16),
@@ -352,12 +407,7 @@ __global__ void attn_schedule_kernel(const int* cu, const int* kv_len, int B, in
   }
 }
 
-}  // namespace
-
-int tc_attn_smem_bytes() { return SMEM_BYTES; }
-
 template <bool F16>
-static
 cudaError_t launch_typed(const CUtensorMap& mQKV, const AttnParams& p, int grid, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
@@ -370,12 +420,13 @@ cudaError_t launch_typed(const CUtensorMap& mQKV, const AttnParams& p, int grid,
   return cudaGetLastError();
 }
 
+}  // namespace
+
+int tc_attn_smem_bytes() { return SMEM_BYTES; }
 
 cudaError_t launch_tc_attn(const CUtensorMap& mQKV, const AttnParams& p, int grid, bool f16, cudaStream_t st) {
   return f16 ? launch_typed<true>(mQKV, p, grid, st) : launch_typed<false>(mQKV, p, grid, st);
 }
-
-
 
 cudaError_t launch_attn_schedule(const int* cu, const int* kv_len, int B, int n_heads, int T_cap, int4* work,
                                  int* work_count, int max_units, int* err, cudaStream_t st) {
