@@ -6,11 +6,15 @@
 // beyond kv_len (bucket padding of the static path) are never keys.
 //
 // One CTA per (segment, head, 128-query tile); 64 + 128 * NGRP threads:
-//   warp 0     TMA producer: Q tile once, then K_j and V_j (128 keys x 128
-//              dims, 128-byte swizzle) into a 2-deep ring;
+//   warp 0     TMA producers: Q once, then K_j (lane 0) and V_j (lane 1),
+//              128 keys x 128 dims with 128-byte swizzle, each in a 3-deep
+//              ring (key tiles take ~2000 cycles to land under load);
 //   warp 1     TMEM allocator + MMA issuer: S_j = Q K_j^T (M=N=128, K=16 x 8)
 //              into one of two S buffers, then O += P_j V_j (V as an MN-major
-//              operand) into the O accumulator;
+//              operand) into the O accumulator.  Q and P are A operands read
+//              from tensor memory, so each MMA streams only its B operand
+//              from shared memory (shared-memory bandwidth bounds an
+//              all-shared-memory version);
 //   warps 2.. softmax, NGRP groups of four warps: a query row (one TMEM
 //              lane) is shared by one thread of each group, which owns
 //              128 / NGRP of the key columns (and of the output dims); the
@@ -18,9 +22,9 @@
 //              once per key tile (an mbarrier, so every wait is bounded).
 //              Online softmax in the log2 domain with lazy rescaling: O is
 //              rescaled in TMEM only when the running max grows by more than
-//              2^8.  P_j goes to shared memory in the swizzled K-major layout
-//              the tensor core reads.
-// The QK^T MMA of tile j+1 overlaps the softmax of tile j.
+//              2^8.  The softmax warps stage Q into tensor memory once and
+//              write each P_j there (tcgen05.st).
+// The QK^T MMAs run up to two key tiles ahead of the softmax.
 // The schedule kernel orders work units longest segment first.
 #include <math.h>
 
@@ -39,14 +43,20 @@ constexpr int SOFTMAX_WARPS = 4 * NGRP;
 constexpr int THREADS = 64 + 32 * SOFTMAX_WARPS;
 constexpr int TILE_BYTES = 128 * DH * 2;   // 32 KB: 128 rows x 128 16-bit values as two 16 KB swizzle panels
 constexpr int PANEL = 16384;
+// Six 32 KB slots: Q in slot 0 (free again once Q sits in tensor memory),
+// K stages 0, 1, 2 in slots 1, 2, 0 and V stages 0, 1, 2 in slots 3, 4, 5.
+constexpr int KV_STAGES = 3;
 constexpr int OFF_Q = 0;
-constexpr int OFF_K = TILE_BYTES;           // 2 buffers
-constexpr int OFF_V = 3 * TILE_BYTES;       // 2 buffers
-constexpr int OFF_P = 5 * TILE_BYTES;
+__host__ __device__ constexpr int k_slot(int st) { return (st == 2 ? 0 : st + 1) * TILE_BYTES; }
+__host__ __device__ constexpr int v_slot(int st) { return (3 + st) * TILE_BYTES; }
 constexpr int OFF_BAR = 6 * TILE_BYTES;
 constexpr int OFF_RED = OFF_BAR + 256;      // float max[2 tiles][NGRP][128] + float sum[NGRP][128]
 constexpr int SMEM_BYTES = OFF_RED + (2 * NGRP * 128 + NGRP * 128) * 4 + 1024;
-constexpr uint32_t TMEM_COLS = 512;         // S0 [0,128), S1 [128,256), O [256,384)
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t TM_O = 256;              // TMEM columns: S0 [0,128), S1 [128,256), O [256,384),
+constexpr uint32_t TM_Q = 384;              //   Q [384,448) and P [448,512) as packed 16-bit pairs
+constexpr uint32_t TM_P = 448;
+static_assert(NGRP == 2, "the TMEM staging of Q and P assumes two 64-column groups");
 constexpr float RESCALE_THRESHOLD = 8.0f;   // log2 units
 
 __device__ __forceinline__ float ex2(float x) {
@@ -74,17 +84,18 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;     // [2]
-  uint64_t* k_empty = bars + 3;    // [2]
-  uint64_t* v_full = bars + 5;     // [2]
-  uint64_t* v_empty = bars + 7;    // [2]
-  uint64_t* s_full = bars + 9;     // [2]
-  uint64_t* s_empty = bars + 11;   // [2]
-  uint64_t* p_full = bars + 13;
-  uint64_t* pv_done = bars + 14;
-  uint64_t* max_ready = bars + 15; // [2] row-max exchange, one per tile parity
-  uint64_t* sum_ready = bars + 17;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+  uint64_t* k_full = bars + 1;     // [KV_STAGES]
+  uint64_t* k_empty = bars + 4;    // [KV_STAGES]
+  uint64_t* v_full = bars + 7;     // [KV_STAGES]
+  uint64_t* v_empty = bars + 10;   // [KV_STAGES]
+  uint64_t* s_full = bars + 13;    // [2]
+  uint64_t* s_empty = bars + 15;   // [2]
+  uint64_t* p_full = bars + 17;
+  uint64_t* pv_done = bars + 18;
+  uint64_t* max_ready = bars + 19; // [2] row-max exchange, one per tile parity
+  uint64_t* sum_ready = bars + 21;
+  uint64_t* q_staged = bars + 22;  // Q copied from shared to tensor memory
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 23);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* red_max = reinterpret_cast<float*>(smem + OFF_RED);   // [2 tiles][NGRP][128] partial row maxima
   float* red_sum = red_max + 2 * NGRP * 128;                   // [NGRP][128] partial row sums
@@ -94,11 +105,13 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < KV_STAGES; ++i) {
       mbar_init(&k_full[i], 1);
       mbar_init(&k_empty[i], 1);
       mbar_init(&v_full[i], 1);
       mbar_init(&v_empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
       mbar_init(&s_empty[i], SOFTMAX_WARPS);
       mbar_init(&max_ready[i], SOFTMAX_WARPS);
@@ -106,6 +119,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(p_full, SOFTMAX_WARPS);
     mbar_init(pv_done, 1);
     mbar_init(sum_ready, SOFTMAX_WARPS);
+    mbar_init(q_staged, SOFTMAX_WARPS);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -116,80 +130,106 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
+    // -------------------------------------------------- TMA producer
+    // lane 0 loads Q and the K tiles, lane 1 the V tiles, so waiting for a V
+    // buffer (freed by PV) never delays the next K (needed by QK^T).
     if (lane == 0) {
-      // ------------------------------------------------ TMA producer
       tma_prefetch_desc(&mQKV);
-      int issued_k = 0, issued_v = 0;
       mbar_arrive_expect_tx(q_full, TILE_BYTES);
       tma_load_2d(smem + OFF_Q, &mQKV, q_full, xq, q0);
       tma_load_2d(smem + OFF_Q + PANEL, &mQKV, q_full, xq + 64, q0);
+    }
+    if (lane < 2) {
+      const bool is_k = lane == 0;
+      uint64_t* full = is_k ? k_full : v_full;
+      uint64_t* empty = is_k ? k_empty : v_empty;
+      const int x = is_k ? xk : xv;
+      int issued = 0;
       for (int j = 0; j < nkv; ++j) {
-        const int sb = j & 1, use = j >> 1;
-        const int row = seq0 + j * BKV;
-        if (use > 0 && !mbar_wait(&k_empty[sb], (use - 1) & 1, abort_flag, p.err)) break;
-        uint8_t* kd = smem + OFF_K + sb * TILE_BYTES;
-        mbar_arrive_expect_tx(&k_full[sb], TILE_BYTES);
-        tma_load_2d(kd, &mQKV, &k_full[sb], xk, row);
-        tma_load_2d(kd + PANEL, &mQKV, &k_full[sb], xk + 64, row);
-        ++issued_k;
-        if (use > 0 && !mbar_wait(&v_empty[sb], (use - 1) & 1, abort_flag, p.err)) break;
-        uint8_t* vd = smem + OFF_V + sb * TILE_BYTES;
-        mbar_arrive_expect_tx(&v_full[sb], TILE_BYTES);
-        tma_load_2d(vd, &mQKV, &v_full[sb], xv, row);
-        tma_load_2d(vd + PANEL, &mQKV, &v_full[sb], xv + 64, row);
-        ++issued_v;
+        const int st = j % KV_STAGES, use = j / KV_STAGES;
+        if (use > 0 && !mbar_wait(&empty[st], (use - 1) & 1, abort_flag, p.err)) break;
+        // K stage 2 reuses Q's slot: wait until Q has been staged in tensor memory
+        if (is_k && j == 2 && !mbar_wait(q_staged, 0, abort_flag, p.err)) break;
+        uint8_t* dst = smem + (is_k ? k_slot(st) : v_slot(st));
+        mbar_arrive_expect_tx(&full[st], TILE_BYTES);
+        tma_load_2d(dst, &mQKV, &full[st], x, seq0 + j * BKV);
+        tma_load_2d(dst + PANEL, &mQKV, &full[st], x + 64, seq0 + j * BKV);
+        ++issued;
       }
       if (*abort_flag) {
-        mbar_wait_drain(q_full, 0, 200000000ull);
-        for (int j = issued_k > 2 ? issued_k - 2 : 0; j < issued_k; ++j)
-          mbar_wait_drain(&k_full[j & 1], (j >> 1) & 1, 200000000ull);
-        for (int j = issued_v > 2 ? issued_v - 2 : 0; j < issued_v; ++j)
-          mbar_wait_drain(&v_full[j & 1], (j >> 1) & 1, 200000000ull);
+        if (is_k) mbar_wait_drain(q_full, 0, 200000000ull);
+        for (int j = issued > KV_STAGES ? issued - KV_STAGES : 0; j < issued; ++j)
+          mbar_wait_drain(&full[j % KV_STAGES], (j / KV_STAGES) & 1, 200000000ull);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------ MMA issuer
+      // Issues QK^T for tile js as soon as K_js has landed and its S buffer is
+      // free (up to two tiles ahead of the softmax), and PV for tile jp as soon
+      // as P_jp is ready; both conditions are polled, never blocked on, so a
+      // slow softmax never holds back the next QK^T.
       constexpr uint32_t idesc_qk = make_idesc(BQ, BKV, 0, F16);
       constexpr uint32_t idesc_pv = make_idesc(BQ, DH, 1, F16);
-      const uint32_t sq = smem_u32(smem + OFF_Q);
-      const uint32_t sp = smem_u32(smem + OFF_P);
-      auto issue_pv = [&](int i) -> bool {
-        const int sb = i & 1, use = i >> 1;
-        if (!mbar_wait(&v_full[sb], use & 1, abort_flag, p.err)) return false;
-        if (!mbar_wait(p_full, i & 1, abort_flag, p.err)) return false;
-        tc_fence_after();
-        const uint32_t sv = smem_u32(smem + OFF_V + sb * TILE_BYTES);
+      bool ok = mbar_wait(q_staged, 0, abort_flag, p.err);
+      int js = 0, jp = 0;
+      uint64_t t_idle = 0;
+      uint32_t spins = 0;
+      while (ok && jp < nkv) {
+        bool progressed = false;
+        if (js < nkv) {
+          const int sb = js & 1, use = js >> 1;
+          const int kst = js % KV_STAGES, kuse = js / KV_STAGES;
+          if (mbar_test_wait(&k_full[kst], kuse & 1) && (use == 0 || mbar_test_wait(&s_empty[sb], (use - 1) & 1))) {
+            tc_fence_after();
+            const uint32_t sk = smem_u32(smem + k_slot(kst));
 #pragma unroll
-        for (int k = 0; k < BKV / 16; ++k) {
-          const uint64_t ad = make_sdesc_sw128(sp + (k >> 2) * PANEL + (k & 3) * 32, 16, 1024);
-          // V is [keys, dims] with dims contiguous: MN-major B operand; the two
-          // 64-dim panels are PANEL bytes apart (LBO), 8-key groups 1 KB apart (SBO)
-          const uint64_t bd = make_sdesc_sw128(sv + k * 16 * 128, PANEL, 1024);
-          tc_mma_f16(tmem + 256, ad, bd, idesc_pv, (i > 0 || k > 0) ? 1u : 0u);
+            for (int k = 0; k < DH / 16; ++k) {
+              // A = Q from tensor memory, B = K_js (K-major, 128-byte swizzle)
+              const uint32_t off = (k >> 2) * PANEL + (k & 3) * 32;
+              tc_mma_f16_tmem_a(tmem + sb * 128, tmem + TM_Q + 8 * k, make_sdesc_sw128(sk + off, 16, 1024), idesc_qk,
+                                k > 0 ? 1u : 0u);
+            }
+            tc_commit(&k_empty[kst]);
+            tc_commit(&s_full[sb]);
+            ++js;
+            progressed = true;
+          }
         }
-        tc_commit(&v_empty[sb]);
-        tc_commit(pv_done);
-        return true;
-      };
-      bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
-      for (int j = 0; ok && j < nkv; ++j) {
-        const int sb = j & 1, use = j >> 1;
-        if (!mbar_wait(&k_full[sb], use & 1, abort_flag, p.err)) { ok = false; break; }
-        if (use > 0 && !mbar_wait(&s_empty[sb], (use - 1) & 1, abort_flag, p.err)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t sk = smem_u32(smem + OFF_K + sb * TILE_BYTES);
+        if (jp < js) {
+          const int vst = jp % KV_STAGES, vuse = jp / KV_STAGES;
+          if (mbar_test_wait(&v_full[vst], vuse & 1) && mbar_test_wait(p_full, jp & 1)) {
+            tc_fence_after();
+            const uint32_t sv = smem_u32(smem + v_slot(vst));
 #pragma unroll
-        for (int k = 0; k < DH / 16; ++k) {
-          const uint32_t off = (k >> 2) * PANEL + (k & 3) * 32;
-          tc_mma_f16(tmem + sb * 128, make_sdesc_sw128(sq + off, 16, 1024), make_sdesc_sw128(sk + off, 16, 1024),
-                     idesc_qk, k > 0 ? 1u : 0u);
+            for (int k = 0; k < BKV / 16; ++k) {
+              // A = P from tensor memory (8 columns per 16 keys); B = V, which is
+              // [keys, dims] with dims contiguous: an MN-major operand whose two
+              // 64-dim panels are PANEL bytes apart (LBO), 8-key groups 1 KB apart (SBO)
+              const uint64_t bd = make_sdesc_sw128(sv + k * 16 * 128, PANEL, 1024);
+              tc_mma_f16_tmem_a(tmem + TM_O, tmem + TM_P + 8 * k, bd, idesc_pv, (jp > 0 || k > 0) ? 1u : 0u);
+            }
+            tc_commit(&v_empty[vst]);
+            tc_commit(pv_done);
+            ++jp;
+            progressed = true;
+          }
         }
-        tc_commit(&k_empty[sb]);
-        tc_commit(&s_full[sb]);
-        if (j > 0 && !issue_pv(j - 1)) { ok = false; break; }
+        if (progressed) {
+          spins = 0;
+        } else if ((++spins & 255u) == 0) {
+          // bounded: give up (and let every role unwind) after the wait limit
+          const uint64_t now = globaltimer_ns();
+          if (t_idle == 0) t_idle = now;
+          if (*abort_flag) break;
+          if (now - t_idle > kWaitLimitNs) {
+            *abort_flag = 1;
+            record_error(p.err, kErrTimeout);
+            break;
+          }
+        }
+        if (progressed) t_idle = 0;
       }
-      if (ok && nkv > 0) issue_pv(nkv - 1);
     }
   } else {
     // -------------------------------------------------- softmax warps 2..
@@ -199,15 +239,27 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int col0 = grp * COLS;
     const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
     const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
-    // P row r, keys [col0, col0 + COLS): 16-byte chunks (col0 % 64) / 8 + c of
-    // panel col0 / 64 in the swizzled K-major layout (chunk k of row r sits at
-    // (r / 8) * 1024 + (r % 8) * 128 + ((k ^ (r % 8)) * 16))
-    uint8_t* sProw = smem + OFF_P + (col0 / 64) * PANEL + (r >> 3) * 1024 + (r & 7) * 128;
-    const int chunk0 = (col0 % 64) / 8;
     float m_ref = -INFINITY;                      // running max, log2 units
     float l = 0.f;                                // partial row sum over this thread's columns
-    bool ok = true;
-    for (int j = 0; j < nkv; ++j) {
+    bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
+    if (ok) {
+      // stage Q row r, dims [col0, col0 + 64) (swizzle panel grp) into tensor
+      // memory: 16-byte chunk c of the row sits at (r / 8) * 1024 + (r % 8) * 128
+      // + ((c ^ (r % 8)) * 16) of the panel
+      const uint8_t* qrow = smem + OFF_Q + grp * PANEL + (r >> 3) * 1024 + (r & 7) * 128;
+      uint32_t qv[32];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        const uint4 v = *reinterpret_cast<const uint4*>(qrow + ((c ^ (r & 7)) * 16));
+        qv[4 * c + 0] = v.x; qv[4 * c + 1] = v.y; qv[4 * c + 2] = v.z; qv[4 * c + 3] = v.w;
+      }
+      tmem_st32(tmem + lane_off + TM_Q + 32 * grp, qv);
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(q_staged);
+    }
+    for (int j = 0; ok && j < nkv; ++j) {
       const int sb = j & 1, use = j >> 1;
       if (!mbar_wait(&s_full[sb], use & 1, abort_flag, p.err)) { ok = false; break; }
       tc_fence_after();
@@ -232,18 +284,17 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int c = 0; c < COLS; ++c) s[c] = c < valid ? s[c] : -INFINITY;
       }
-      // tree-shaped max over this group's columns, then exchange with the
+      // pairwise max tree over this group's columns, then exchange with the
       // other groups of the row (double-buffered by tile parity, bounded wait)
-      float mx[8];
+      float mx[COLS / 2];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mx[i] = s[i];
+      for (int i = 0; i < COLS / 2; ++i) mx[i] = fmaxf(s[2 * i], s[2 * i + 1]);
 #pragma unroll
-      for (int c = 8; c < COLS; c += 8) {
+      for (int w = COLS / 4; w >= 1; w >>= 1) {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx[i] = fmaxf(mx[i], s[c + i]);
+        for (int i = 0; i < w; ++i) mx[i] = fmaxf(mx[i], mx[i + w]);
       }
-      const float mloc = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      const float mloc = mx[0];
       float* rm = red_max + (j & 1) * (NGRP * 128);
       rm[grp * 128 + r] = mloc;
       __syncwarp();
@@ -276,12 +327,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         // last, partial key tile: groups 0 and 1 clear value panels 0 and 1
         // of the rows past kv_len so stale (possibly non-finite) data cannot
         // meet the zero probabilities
-        if (!mbar_wait(&v_full[sb], use & 1, abort_flag, p.err)) { ok = false; break; }
+        const int vst = j % KV_STAGES;
+        if (!mbar_wait(&v_full[vst], (j / KV_STAGES) & 1, abort_flag, p.err)) { ok = false; break; }
         if (r >= valid_all) {
-          uint4* v = reinterpret_cast<uint4*>(smem + OFF_V + sb * TILE_BYTES + grp * PANEL + r * 128);
+          uint4* v = reinterpret_cast<uint4*>(smem + v_slot(vst) + grp * PANEL + r * 128);
 #pragma unroll
           for (int i = 0; i < 8; ++i) v[i] = make_uint4(0, 0, 0, 0);
         }
+        fence_proxy_async_smem();
       }
       if (j > 0) {
         if (!mbar_wait(pv_done, (j - 1) & 1, abort_flag, p.err)) { ok = false; break; }
@@ -300,12 +353,9 @@ __global__ void __launch_bounds__(THREADS, 1)
           tmem_st_wait();
         }
       }
-#pragma unroll
-      for (int c = 0; c < COLS / 8; ++c) {
-        uint4* dst = reinterpret_cast<uint4*>(sProw + (((chunk0 + c) ^ (r & 7)) * 16));
-        *dst = make_uint4(pk[4 * c + 0], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-      }
-      fence_proxy_async_smem();
+      // this thread's keys of row r -> P in tensor memory (packed pairs)
+      tmem_st32(tmem + lane_off + TM_P + 32 * grp, pk);
+      tmem_st_wait();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full);
