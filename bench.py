@@ -59,6 +59,24 @@ def peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
+def measured_traffic(workload: int, kernel: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu capture of this
+    workload, or None when the kernel sources changed since that capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"traffic_workload{workload}.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        doc = json.load(f)
+    h = hashlib.sha1()
+    for s in doc["sources"]:
+        with open(os.path.join(ROOT, s), "rb") as f:
+            h.update(f.read())
+    if h.hexdigest() != doc["sources_sha1"] or kernel not in doc["kernels"]:
+        return None
+    return doc["kernels"][kernel]["traffic_bytes"]
+
+
 def layer_flops(seg, kv, d, F):
     """Algorithmic FLOPs of one layer (Eq. 2 made exact): projections 8*T*d^2,
     MLP 6*T*d*F, attention 4*d*sum(L_q * L_kv)."""
@@ -434,7 +452,9 @@ def main():
     achieved = gu.get("tflops")
     peak = pk["bf16_tflops_sustained"]
     roofline = {"kernel": "tc_gemm_kernel<Swiglu> (gate/up + SwiGLU)", "bound": "tensor", "achieved": achieved,
-                "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak if achieved else None, "traffic": None,
+                "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak if achieved else None,
+                "traffic": measured_traffic(wl.index, "gate_up"),
+                "algorithmic_bytes": float(2 * T_exec * d + 2 * 2 * F * d + 2 * T_exec * F),
                 "peak_source": f"{src} bf16 dense, sustained (f16 operands run at the bf16 rate)",
                 "flops_per_launch": flops_of["gate_up"]}
 

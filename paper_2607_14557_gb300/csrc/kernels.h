@@ -36,6 +36,7 @@ struct GemmParams {
   uint32_t idesc;         // tcgen05 instruction descriptor (operand type f16 or bf16)
   int out_type;           // ElemType of C (kBF16 / kF16; kF32 on the CUDA-core path)
   int res_type;           // ElemType of R
+  int group_m;            // raster: m-tiles per group (see tc_gemm.cu)
 };
 
 struct AttnParams {

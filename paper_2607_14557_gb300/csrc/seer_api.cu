@@ -87,6 +87,19 @@ bool is16(seer_dtype dt) { return dt == SEER_BF16 || dt == SEER_F16; }
 size_t esize(seer_dtype dt) { return dt == SEER_F32 ? 4 : 2; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// L2 raster of the tcgen05 GEMM: keep the whole weight operand resident when
+// it is at most 40 MB (group_m = 1, n varies fastest), otherwise keep about
+// 24 MB of 128-row slabs of A resident while the weights stream past them.
+// Both budgets come from a sweep on GB300 at the 8B layer shapes (larger A
+// slabs thrash the L2 and re-read more, smaller ones re-stream the weights).
+int gemm_group_m(long b_bytes, long a_tile_bytes) {
+  constexpr long kResident = 40l << 20;
+  constexpr long kBudget = 24l << 20;
+  if (b_bytes <= kResident) return 1;
+  const long g = kBudget / (a_tile_bytes > 0 ? a_tile_bytes : 1);
+  return static_cast<int>(g < 1 ? 1 : (g > 4096 ? 4096 : g));
+}
+
 // ------------------------------------------------------------ TMA descriptors
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
@@ -238,6 +251,7 @@ seer_status do_linear(const void* a, const void* w, seer_dtype op_dt, const void
       return fail(SEER_ERR_UNSUPPORTED, "16-bit linear needs 16-byte aligned pointers");
     if (M_cap == 0) return SEER_OK;
     p.idesc = make_idesc(128, 256, 0, op_dt == SEER_F16);
+    p.group_m = gemm_group_m(2l * N * K, 2l * 128 * K);
     CUtensorMap mA, mB;
     SEER_TRY(make_map16(&mA, a, op_dt, M_cap, K, K, 128));
     SEER_TRY(make_map16(&mB, w, op_dt, N, K, K, 128));
@@ -293,6 +307,7 @@ seer_status do_swiglu(const void* a, const void* wg, const void* wu, seer_dtype 
   if (M_cap == 0) return SEER_OK;
   if (is16(op_dt)) {
     p.idesc = make_idesc(128, 256, 0, op_dt == SEER_F16);
+    p.group_m = gemm_group_m(2l * 2 * F * K, 2l * 128 * K);
     CUtensorMap mA, mG, mU;
     SEER_TRY(make_map16(&mA, a, op_dt, M_cap, K, K, 128));
     SEER_TRY(make_map16(&mG, wg, op_dt, F, K, K, 128));

@@ -36,16 +36,19 @@ constexpr int STAGE_BYTES = A_TILE_BYTES + 2 * B_HALF_BYTES;  // 48 KB
 constexpr int THREADS = 192;
 constexpr int ACC_COLS = 256;
 constexpr int TMEM_COLS = 512;
-constexpr int GROUP_M = 16;                          // m-tiles per raster group (L2 reuse)
 constexpr int BAR_BYTES = 256;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
 
-__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int& m, int& n) {
-  const int per_group = GROUP_M * num_n;
+// Raster: groups of `group_m` m-tiles; inside a group m varies fastest and
+// the group sweeps every n-tile.  group_m = 1 keeps the whole B operand hot in
+// L2 while A streams once; a large group_m keeps a slab of A hot while B
+// streams once per group (chosen on the host from the operand sizes).
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group_m, int& m, int& n) {
+  const int per_group = group_m * num_n;
   const int g = t / per_group;
   const int r = t - g * per_group;
-  const int m0 = g * GROUP_M;
-  const int gm = min(GROUP_M, num_m - m0);
+  const int m0 = g * group_m;
+  const int gm = min(group_m, num_m - m0);
   m = m0 + r % gm;
   n = r / gm;
 }
@@ -90,6 +93,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int num_n = halfN ? p.N / 128 : p.N / BN;
   const int num_tiles = num_m * num_n;
   const int KB = p.K / BK;
+  const int group_m = p.group_m > 0 ? p.group_m : 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -120,7 +124,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       long issued = 0;
       for (int t = blockIdx.x; t < num_tiles && !*abort_flag; t += gridDim.x) {
         int m, n;
-        tile_coords(t, num_m, num_n, m, n);
+        tile_coords(t, num_m, num_n, group_m, m, n);
         int a_row;
         if (MODE == kGemmCount) {
           const int b = m / tiles_per_seq;
@@ -194,7 +198,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t acc_ph = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
       int m, n;
-      tile_coords(t, num_m, num_n, m, n);
+      tile_coords(t, num_m, num_n, group_m, m, n);
       if (!mbar_wait(&acc_full[acc], acc_ph, abort_flag, p.err)) break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + lane_off + static_cast<uint32_t>(acc * ACC_COLS);
