@@ -1,6 +1,6 @@
 """fp64 numpy oracle of the Seer hot path.  Test infrastructure only.
 
-Readings of the paper that this file takes (each also listed in the design doc):
+Readings of the paper that this file takes:
 
 * The "MLP activation" whose sparsity is measured is the SwiGLU intermediate
   ``a = SiLU(x Wg^T) * (x Wu^T)`` (the input of the down projection); a value
