@@ -247,12 +247,16 @@ def run_stack(args, wl, world, rank, local):
         for _ in range(n_steps):
             g_pad.replay()
         ev[3].record(stream)
+        stack.step0_truncating(x_full, cu_full, resp, ctx, stream)
+        ev[4].record(stream)
         torch.cuda.synchronize()
     assert S.seer_check_device() == 0
     ms0 = ev[0].elapsed_time(ev[1])
     ms_rest = ev[1].elapsed_time(ev[2])
     ms_pad = ev[2].elapsed_time(ev[3])
     ms_seer = ms0 + ms_rest
+    ms0_f1 = ev[3].elapsed_time(ev[4])
+    dl = detect_layer + 1
     fl_full = layer_flops(lens.full, lens.full, d, F) * nl
     fl_trunc = layer_flops(seg, kv, d, F) * nl
     fl_valid = layer_flops(kv, kv, d, F) * nl
@@ -276,7 +280,12 @@ def run_stack(args, wl, world, rank, local):
                   "tflops_truncated_steps": tflops_rest, "frac_of_burst_peak": tflops_rest / pk["bf16_tflops"],
                   "tflops_padded": fl_full * n_steps / (ms_pad * 1e-3) / 1e12,
                   "truncated_tokens_per_s": T_valid * nl * (n_steps - 1) / (ms_rest * 1e-3)},
-        "gpu_launches": nl * 8 * (2 * n_steps) + 3, "clocks": clk.summary(),
+        "step0_truncated_after_detection": {
+            "ms_step0": ms0_f1, "layers_full": dl, "layers_packed": nl - dl,
+            "ms_total_%d_steps" % n_steps: ms0_f1 + ms_rest, "speedup_vs_padded": ms_pad / (ms0_f1 + ms_rest),
+            "ideal_ratio": fl_full * n_steps / (fl_full * dl / nl + fl_valid * (nl - dl) / nl + fl_valid * (n_steps - 1)),
+            "tokens_per_s": (T_full * dl + T_valid * (nl - dl) + (n_steps - 1) * T_valid * nl) / ((ms0_f1 + ms_rest) * 1e-3)},
+        "gpu_launches": nl * 8 * (2 * n_steps) + 3 + (nl * 8 + 4), "clocks": clk.summary(),
         "peak_source": src,
     }
     if rank == 0:
@@ -398,6 +407,14 @@ def main():
 
     ms_layer = timed(lambda: path.layer(W, stream=stream), args.steps)
     ms_pad = timed(lambda: path.padded_forward(x_full, cu_full, W, y_full, stream), args.steps)
+    # naive-pad comparator: truncated sequences padded to the batch's longest L* (keys masked)
+    x_nv, cu_nv, kv_nv, T_nv = path.naive_pad_inputs(x_full, cu_full, ctx, stream)
+    y_nv = torch.empty((T_nv, d), dtype=tdt, device=dev)
+    ms_naive = timed(lambda: path.layer(W, x=x_nv, y=y_nv, cu=cu_nv, kv=kv_nv, T_cap=T_nv, stream=stream),
+                     args.steps)
+    seg_nv = np.diff(cu_nv.cpu().numpy())
+    flops_naive = layer_flops(seg_nv, kv_nv.cpu().numpy(), d, F)
+    del x_nv, y_nv
 
     # ---- end to end through the API with host buffers
     e2e = None
@@ -477,6 +494,8 @@ def main():
                   "frac_of_sustained_peak": flops_exec / (ms_layer * 1e-3) / 1e12 / pk["bf16_tflops_sustained"],
                   "speedup_vs_padded": ms_pad / ms_layer, "ideal_ratio": flops_pad / flops_valid,
                   "flops_executed": flops_exec, "flops_valid": flops_valid, "flops_padded": flops_pad},
+        "naive_pad": {"ms": ms_naive, "tokens_executed": int(T_nv), "flops_executed": flops_naive,
+                      "speedup_truncated_vs_naive": ms_naive / ms_layer, "ideal_ratio": flops_naive / flops_valid},
         "speedup_step_vs_padded_layer": ms_pad / ms_step,
         "kernels": kernels, "roofline": roofline, "gpu_launches": KERNELS_PER_STEP * args.steps,
         "e2e": e2e, "clocks": clocks,

@@ -142,6 +142,34 @@ class SeerPath:
         return {"total": int(c[1]), "max_seqlen": int(c[2]), "capacity": int(c[3]), "path_mask": int(c[5]),
                 "pad_rows": int(c[6]), "groups": groups}
 
+    def naive_pad_inputs(self, x_full, cu_full, ctx_len, stream=None):
+        """Inputs of the naive-pad comparator (the batch-max padding that Sec. 3.4
+        improves on, Eq. 3): every sequence keeps ``ctx_b + max_b L*_b`` rows,
+        rows past ``ctx_b + L*_b`` are computed as queries and masked as keys.
+
+        Built once after a step has produced ``L_star`` (reads it on the host);
+        the rows are gathered by the library's pack kernel with the static path
+        switched off (``tau_pad < 0``), so every segment keeps exactly its rows.
+        Returns ``(x, cu, kv_len, T)``.
+        """
+        B, dev = self.B, self.device
+        L = self.L_star.cpu().numpy().astype(np.int64)
+        ctx = ctx_len.cpu().numpy().astype(np.int64)
+        L_max = int(L.max())
+        T = int(ctx.sum() + B * L_max)
+        i32 = dict(dtype=torch.int32, device=dev)
+        L_pad = torch.full((B,), L_max, **i32)
+        x = torch.zeros((max(T, 1), self.dims.d_model), dtype=self.x_packed.dtype, device=dev)
+        cu = torch.empty(B + 1, **i32)
+        kv_all = torch.empty(B, **i32)
+        meta = torch.empty(S.CTRL_WORDS, **i32)
+        p = self.params
+        no_static = S.make_params(p.act_eps, p.tau_jump, p.gamma, p.window, -1.0, p.eager_max_bucket)
+        S.seer_pack_ragged(x_full, self.dtype, cu_full, ctx_len, L_pad, B, self.dims.d_model, self.N, T, no_static, x,
+                           cu, kv_all, meta, None, 0, stream=stream)
+        kv = torch.as_tensor((ctx + L).astype(np.int32)).to(dev)
+        return x, cu, kv, T
+
     def padded_forward(self, x_full, cu_full, w: LayerWeights, y_full, stream=None):
         """The same layer over the untruncated windows (every key kept)."""
         S.seer_layer_forward(w.struct(), self.dims, self.dtype, x_full, y_full, cu_full, None, self.B, self.T_full,
@@ -174,11 +202,14 @@ class SeerStack:
         self.buf = [torch.empty((T_full, d), dtype=tdt, device=dev) for _ in range(2)]
         self.hook_counts = torch.zeros(B * N, dtype=torch.int32, device=dev)
         self.graphs: Dict[object, torch.cuda.CUDAGraph] = {}
+        self.h_packed: Optional[torch.Tensor] = None
 
-    def _run_layers(self, x, cu, kv, T_cap, resp_start=None, stream=None, n_layers=None):
+    def _run_layers(self, x, cu, kv, T_cap, resp_start=None, stream=None, n_layers=None, start=0):
         p = self.path
         cur = x
-        for li, w in enumerate(self.layers[:n_layers]):
+        stop = len(self.layers) if n_layers is None else n_layers
+        for li in range(start, stop):
+            w = self.layers[li]
             out = self.buf[li % 2] if cur is not self.buf[li % 2] else self.buf[(li + 1) % 2]
             count = resp_start is not None and li == self.detect_layer
             S.seer_layer_forward(w.struct(), p.dims, p.dtype, cur, out, cu, kv, p.B, T_cap,
@@ -195,6 +226,25 @@ class SeerStack:
         p.detect(x_full, resp_start, self.layers[self.detect_layer], stream)
         p.pack(x_full, cu_full, ctx_len, stream)
         return out
+
+    def step0_truncating(self, x_full, cu_full, resp_start, ctx_len, stream=None):
+        """Step 0 truncated inside the step (Sec. 3.1: the layers after detection
+        run on the retained tokens only): layers ``0..detect_layer`` over the
+        full windows with the count hook, detection and route/pack, then the
+        detection layer's output is compacted with the same layout and the
+        remaining layers run over the packed sequences.  The step-0 input is
+        packed too (input of the later steps).  Returns the last layer's output
+        in the packed layout."""
+        p = self.path
+        h = self._run_layers(x_full, cu_full, None, p.T_full, resp_start=resp_start, stream=stream,
+                             n_layers=self.detect_layer + 1)
+        p.detect(x_full, resp_start, self.layers[self.detect_layer], stream)
+        p.pack(x_full, cu_full, ctx_len, stream)
+        if self.h_packed is None:
+            self.h_packed = torch.empty_like(p.x_packed)
+        S.seer_pack_ragged(h, p.dtype, cu_full, ctx_len, p.L_star, p.B, p.dims.d_model, p.N, p.T_full, p.params,
+                           self.h_packed, p.cu, p.kv, p.meta, None, 0, stream=stream)
+        return self._run_layers(self.h_packed, p.cu, p.kv, p.T_full, stream=stream, start=self.detect_layer + 1)
 
     def truncated_step(self, T_cap=None, stream=None):
         p = self.path

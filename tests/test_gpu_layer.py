@@ -135,3 +135,37 @@ def test_layer_count_hook_on_full_window():
         parts = oracle.layer_forward_segment(seg, w, wl.n_heads, count_rows=rows, act_eps=0.05, return_parts=True)
         assert np.abs(got[b] - parts["counts"]).max() <= 0.005 * F
         check_close(yh[cu_full[b]:cu_full[b + 1]], parts["y"], "bf16", "full window layer")
+
+
+def test_naive_pad_comparator_matches_truncated_rows():
+    # naive-pad comparator (Eq. 3 batch-max padding): every sequence keeps ctx_b + max L* rows,
+    # the padding is masked as keys, so the valid rows equal the truncated path's rows bit for bit
+    from paper_2607_14557_gb300 import driver as D
+    wl = synth.tiny_workload(dtype="bf16", seed=340, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4, window=160,
+                             boundary=("uniform", 8, 150))
+    lens = synth.lengths(wl)
+    x, cu_full, resp = synth.hidden_full(wl, lens)
+    w = synth.layer_weights(wl, 0)
+    B, N, d = wl.batch, wl.window, wl.d
+    dims = S.make_dims(d, wl.n_heads, wl.head_dim, wl.d_ff)
+    W = D.LayerWeights.from_host(w, "bf16")
+    path = D.SeerPath(dims, "bf16", B, N, x.shape[0], S.make_params(wl.act_eps))
+    xd, cuf, ctx = to_dev(x, "bf16"), i32(cu_full), i32(lens.ctx)
+    path.step(xd, cuf, i32(resp), ctx, W)
+    torch.cuda.synchronize()
+    L = path.L_star.cpu().numpy()
+    np.testing.assert_array_equal(L, lens.boundary + 1)
+    xn, cun, kvn, T = path.naive_pad_inputs(xd, cuf, ctx)
+    yn = torch.full((T, d), 9.0, dtype=torch.bfloat16, device=cuda())
+    path.layer(W, x=xn, y=yn, cu=cun, kv=kvn, T_cap=T)
+    torch.cuda.synchronize()
+    seg = lens.ctx + L.max()
+    cun_h = cun.cpu().numpy()
+    np.testing.assert_array_equal(cun_h, np.concatenate([[0], np.cumsum(seg)]))
+    np.testing.assert_array_equal(kvn.cpu().numpy(), lens.ctx + L)
+    np.testing.assert_array_equal(host(xn), oracle.pack_rows(x, cu_full, seg))
+    cu_t, yt, ynh = path.cu.cpu().numpy(), host(path.y), host(yn)
+    for b in range(B):
+        n = int(lens.ctx[b] + L[b])
+        np.testing.assert_array_equal(ynh[cun_h[b]:cun_h[b] + n], yt[cu_t[b]:cu_t[b] + n])
+    assert np.isfinite(ynh).all()

@@ -1,10 +1,10 @@
 """Workload 3 (32-layer stack, batch 8, 2916+96 context rows, window 512) at full
-batch and sequence sizes, on the first four layers of the stack (each layer
-runs the same launches; depth only repeats them).
+batch, sequence and depth sizes.
 
 Gated against the oracle: boundaries and packing (exact), per-layer outputs of
-layers 0 and 3 on sampled rows (|err| <= 1e-2 + 1e-2|ref|), and the step-0
-count hook (within 0.5% of F).  Properties: a graph-replayed truncated step is
+layers 0 and 3 on sampled rows (|err| <= 1e-2 + 1e-2|ref|), layers 15 and 31
+of a truncated step teacher-forced (the oracle reads the GPU's bf16 input to
+that layer; same bar), and the step-0 count hook (within 0.5% of F).  Properties: a graph-replayed truncated step is
 bit-identical to the eager one.  The two-layer chain is compared with an
 unrounded fp64 chain under three times the one-layer tolerance: the error that
 enters layer 2 (one layer's tolerance plus the bf16 rounding of the stored
@@ -24,7 +24,7 @@ from tests.helpers import check_close, host, i32
 pytestmark = pytest.mark.gpu
 
 S = pytest.importorskip("paper_2607_14557_gb300.seer")
-DEPTH = 4
+DEPTH = 32
 DETECT = 3
 
 
@@ -101,6 +101,25 @@ def test_stack_layer_outputs_sampled_rows(st, layer):
         check_close(y[cu[b] + np.asarray(rows)], ref, "bf16", f"stack layer {layer} segment {b}")
 
 
+@pytest.mark.parametrize("layer", [15, 31])
+def test_stack_teacher_forced_deep_layer(st, layer):
+    wl, stack = st["wl"], st["stack"]
+    p = stack.path
+    x_in = stack._run_layers(p.x_packed, p.cu, p.kv, p.T_full, n_layers=layer).clone()
+    p.layer(stack.layers[layer], x=x_in)
+    torch.cuda.synchronize()
+    y, xh = host(p.y), host(x_in)
+    seg, kv, cu = _segments(st)
+    assert np.isfinite(xh[:cu[-1]]).all()
+    w = synth.layer_weights(wl, layer)
+    rng = np.random.default_rng(100 + layer)
+    for b in (int(np.argmin(seg)), int(np.argmax(seg))):
+        L = int(seg[b])
+        rows = sorted({0, L - 1, int(st["lens"].ctx[b]), *map(int, rng.integers(0, L, 20))})
+        ref = oracle.layer_forward_rows(xh[cu[b]:cu[b + 1]], w, wl.n_heads, rows, kv_len=int(kv[b]))
+        check_close(y[cu[b] + np.asarray(rows)], ref, "bf16", f"stack layer {layer} (teacher-forced) segment {b}")
+
+
 def test_stack_count_hook_matches_oracle(st):
     # the fused hook, moved to layer 0 for this check (same epilogue at any depth)
     wl, stack = st["wl"], st["stack"]
@@ -139,3 +158,32 @@ def test_stack_two_layer_chain_drift(st):
     err = np.abs(got - ref)
     # the bf16 layer boundary is the only extra rounding: three times the one-layer bar
     assert (err <= 3e-2 + 3e-2 * np.abs(ref)).all(), float(err.max())
+
+
+def test_step0_truncated_after_detection_layer(st):
+    # Sec. 3.1 scope: step 0's layers after the detection layer run on the retained tokens only
+    wl, stack = st["wl"], st["stack"]
+    p = stack.path
+    cu_full, resp = st["cu_full"], st["resp"]
+    h_full = stack._run_layers(st["xd"], i32(cu_full), None, p.T_full, n_layers=DETECT + 1).clone()
+    out = stack.step0_truncating(st["xd"], i32(cu_full), i32(resp), i32(st["lens"].ctx))
+    torch.cuda.synchronize()
+    L = p.L_star.cpu().numpy()
+    np.testing.assert_array_equal(L, st["lens"].boundary + 1)
+    seg, kv, cu = _segments(st)
+    T = int(cu[-1])
+    hp = host(stack.h_packed)
+    # the detection layer's full-window output, compacted with the truncated layout (bit exact)
+    np.testing.assert_array_equal(hp[:T], oracle.pack_rows(host(h_full), cu_full, seg))
+    assert np.isfinite(host(out)[:T]).all()
+    # the first packed layer of step 0, teacher-forced on its compacted input
+    nxt = DETECT + 1
+    p.layer(stack.layers[nxt], x=stack.h_packed)
+    torch.cuda.synchronize()
+    y = host(p.y)
+    w = synth.layer_weights(wl, nxt)
+    rng = np.random.default_rng(5)
+    b = int(np.argmin(seg))
+    rows = sorted({0, int(seg[b]) - 1, int(st["lens"].ctx[b]), *map(int, rng.integers(0, int(seg[b]), 20))})
+    ref = oracle.layer_forward_rows(hp[cu[b]:cu[b + 1]], w, wl.n_heads, rows, kv_len=int(kv[b]))
+    check_close(y[cu[b] + np.asarray(rows)], ref, "bf16", "step-0 layer after detection")
