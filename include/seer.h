@@ -56,15 +56,17 @@ typedef enum { SEER_F32 = 0, SEER_BF16 = 1, SEER_F16 = 2 } seer_dtype;
 /* Layer geometry.  A pre-norm block: RMSNorm -> QKV -> bidirectional MHA ->
  * O projection + residual -> RMSNorm -> SwiGLU MLP + residual.  The paper
  * does not spell out the block (it evaluates LLaDA-style backbones); this
- * LLaMA-style reading uses no biases and no positional rotation
- * (rope_theta must be 0). */
+ * LLaMA-style reading uses no biases.  The paper names no positional scheme:
+ * rope_theta > 0 turns on a rotary embedding of q and k (half-split pairs
+ * (i, i + dh/2) rotated by pos * rope_theta^(-2i/dh), pos = the row's index
+ * in its sequence, restarting at 0 in every segment); 0 leaves it off. */
 typedef struct {
   int d_model;
   int n_heads;
   int head_dim;      /* d_model == n_heads * head_dim */
   int d_ff;          /* SwiGLU intermediate width F */
   float rms_eps;     /* 1e-5 */
-  float rope_theta;  /* must be 0 (no rotation) */
+  float rope_theta;  /* 0 = no rotation; > 0 = rotary base (e.g. 10000) */
 } seer_dims;
 
 /* Detector and routing parameters (Sec. 3.3-3.4; defaults in brackets). */
@@ -220,6 +222,16 @@ seer_status seer_rmsnorm(const void* x, seer_dtype x_dt, const void* g, void* y,
  * (N % 256 == 0, K % 64 == 0); with fp32 operands everything is fp32. */
 seer_status seer_linear(const void* a, const void* w, seer_dtype op_dt, const void* r, seer_dtype r_dt, void* c,
                         seer_dtype c_dt, int M_cap, const int32_t* M_dev, int N, int K, void* stream);
+
+/* In-place rotary embedding of the q and k heads of qkv [T, 3*H*dh]
+ * (q | k | v column blocks, any dtype), as seer_layer_forward applies it when
+ * rope_theta > 0 (there fused into the QKV projection's epilogue for 16-bit
+ * layers): pair (i, i + dh/2) of a head turns by pos * theta^(-2i/dh), pos =
+ * row - cu_seqlens[b] for the segment b holding the row.  Rows past
+ * cu_seqlens[B] (device) are untouched.  theta > 0, head_dim even and <= 128.
+ * Not from the paper (which names no positional scheme). */
+seer_status seer_rope(void* qkv, seer_dtype dt, const int32_t* cu_seqlens, int B, int T_capacity, int n_heads,
+                      int head_dim, float theta, void* stream);
 
 /* act[M, F] = SiLU(a w_gate^T) * (a w_up^T) (F % 128 == 0 for 16-bit
  * operands); near-zero counts as in seer_layer_forward. */

@@ -18,7 +18,9 @@ Readings of the paper that this file takes:
   sequences sharing a bucket (Sec. 3.4).
 * The block is a pre-norm LLaMA-style layer (RMSNorm, eps 1e-5; MHA without
   bias; SwiGLU MLP), attention scaled by ``1/sqrt(head_dim)`` (Eq. 7 prints
-  ``sqrt(d)``, read as the per-head width), no positional rotation.
+  ``sqrt(d)``, read as the per-head width).  The paper names no positional
+  scheme; a rotary embedding of queries and keys is optional (off unless
+  ``rope_theta > 0``), positions restarting at 0 in every sequence.
 * A "BF16 layer" stores every tensor that crosses an op boundary in bf16:
   ``xn, q, k, v, o, h, hn, a, y`` are rounded to the storage type after being
   computed exactly (fp64) from already-rounded inputs.
@@ -33,7 +35,7 @@ import numpy as np
 __all__ = [
     "round_bf16", "round_f32", "rounding_for", "silu", "swiglu_activation", "sparsity_counts",
     "snr_boundary", "snr_boundaries", "bucket_set", "bucket_of", "padding_waste_ratio", "route",
-    "segment_layout", "pack_rows", "rmsnorm", "attention_weights", "attention", "layer_forward_segment",
+    "segment_layout", "pack_rows", "rmsnorm", "rope", "attention_weights", "attention", "layer_forward_segment",
     "layer_forward_packed", "layer_forward_rows", "PATH_STATIC", "PATH_VARLEN", "PATH_EAGER",
 ]
 
@@ -212,6 +214,30 @@ def rmsnorm(x, g, eps: float = 1e-5) -> np.ndarray:
     return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * np.asarray(g, dtype=np.float64)
 
 
+def rope(x, positions, n_heads: int, theta: float) -> np.ndarray:
+    """Rotary position embedding of every head of ``x`` [L, H*dh].
+
+    Not from the paper (which names no positional scheme): the rotation of
+    RoFormer (Su et al., 2021) in the half-split layout of LLaMA checkpoints.
+    Pair ``i < dh/2`` of a head is ``(x_i, x_{i+dh/2})``; it is rotated by
+    the angle ``pos * theta^(-2i/dh)``.  ``theta <= 0`` leaves ``x`` as is.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    if theta <= 0:
+        return x.copy()
+    dh = x.shape[1] // n_heads
+    half = dh // 2
+    ang = np.asarray(positions, dtype=np.float64)[:, None] * float(theta) ** (-2.0 * np.arange(half) / dh)
+    c, s = np.cos(ang), np.sin(ang)
+    out = np.empty_like(x)
+    for h in range(n_heads):
+        a = x[:, h * dh:h * dh + half]
+        b = x[:, h * dh + half:(h + 1) * dh]
+        out[:, h * dh:h * dh + half] = a * c - b * s
+        out[:, h * dh + half:(h + 1) * dh] = b * c + a * s
+    return out
+
+
 def attention_weights(q, k) -> np.ndarray:
     """Eqs. 6-7: A[i, j] = exp(e_ij) / sum_u exp(e_iu), e_ij = q_i . k_j / sqrt(dh).
 
@@ -244,21 +270,22 @@ def _f64(a):
 
 def layer_forward_segment(x, w: Dict[str, np.ndarray], n_heads: int, *, kv_len: Optional[int] = None,
                           dtype: Optional[str] = None, rms_eps: float = 1e-5, count_rows=None,
-                          act_eps: float = 0.0, return_parts: bool = False):
+                          act_eps: float = 0.0, return_parts: bool = False, rope_theta: float = 0.0):
     """One pre-norm block over one sequence (Eq. 9-10: keys = retained rows).
 
     ``x`` [L, d] rows of one sequence.  Only the first ``kv_len`` rows serve
     as keys/values (the rest are bucket padding); every row is a query.
     ``count_rows``: optional row indices whose SwiGLU activations are counted
-    against ``act_eps`` (the step-0 detection hook).
+    against ``act_eps`` (the step-0 detection hook).  ``rope_theta > 0``
+    rotates q and k (:func:`rope`) at their row positions in the sequence.
     """
     R = rounding_for(dtype)
     x = _f64(x)
     L = x.shape[0]
     kv = L if kv_len is None else int(kv_len)
     xn = R(rmsnorm(x, w["g_attn"], rms_eps))
-    q = R(xn @ _f64(w["wq"]).T)
-    k = R(xn[:kv] @ _f64(w["wk"]).T)
+    q = R(rope(xn @ _f64(w["wq"]).T, np.arange(L), n_heads, rope_theta))
+    k = R(rope(xn[:kv] @ _f64(w["wk"]).T, np.arange(kv), n_heads, rope_theta))
     v = R(xn[:kv] @ _f64(w["wv"]).T)
     o = R(attention(q, k, v, n_heads))
     h = R(x + o @ _f64(w["wo"]).T)
@@ -274,7 +301,8 @@ def layer_forward_segment(x, w: Dict[str, np.ndarray], n_heads: int, *, kv_len: 
     return (y, counts) if count_rows is not None else y
 
 
-def layer_forward_packed(x_packed, cu, w, n_heads: int, *, kv_len=None, dtype=None, rms_eps=1e-5):
+def layer_forward_packed(x_packed, cu, w, n_heads: int, *, kv_len=None, dtype=None, rms_eps=1e-5,
+                         rope_theta: float = 0.0):
     """Apply :func:`layer_forward_segment` to each packed segment independently."""
     x_packed = _f64(x_packed)
     y = np.empty_like(x_packed)
@@ -282,11 +310,12 @@ def layer_forward_packed(x_packed, cu, w, n_heads: int, *, kv_len=None, dtype=No
         a, b = int(cu[i]), int(cu[i + 1])
         if b > a:
             y[a:b] = layer_forward_segment(x_packed[a:b], w, n_heads, dtype=dtype, rms_eps=rms_eps,
-                                           kv_len=None if kv_len is None else int(kv_len[i]))
+                                           kv_len=None if kv_len is None else int(kv_len[i]), rope_theta=rope_theta)
     return y
 
 
-def layer_forward_rows(x_seg, w, n_heads: int, rows, *, kv_len=None, dtype=None, rms_eps=1e-5, act_eps=None):
+def layer_forward_rows(x_seg, w, n_heads: int, rows, *, kv_len=None, dtype=None, rms_eps=1e-5, act_eps=None,
+                       rope_theta: float = 0.0):
     """Outputs of selected rows of one segment (keys/values from all kept rows).
 
     Same arithmetic as :func:`layer_forward_segment`, restricted to the query
@@ -299,11 +328,11 @@ def layer_forward_rows(x_seg, w, n_heads: int, rows, *, kv_len=None, dtype=None,
     kv = x.shape[0] if kv_len is None else int(kv_len)
     rows = np.asarray(rows, dtype=np.int64)
     xn_kv = R(rmsnorm(x[:kv], w["g_attn"], rms_eps))
-    k = R(xn_kv @ _f64(w["wk"]).T)
+    k = R(rope(xn_kv @ _f64(w["wk"]).T, np.arange(kv), n_heads, rope_theta))
     v = R(xn_kv @ _f64(w["wv"]).T)
     xr = x[rows]
     xn = R(rmsnorm(xr, w["g_attn"], rms_eps))
-    q = R(xn @ _f64(w["wq"]).T)
+    q = R(rope(xn @ _f64(w["wq"]).T, rows, n_heads, rope_theta))
     o = R(attention(q, k, v, n_heads))
     h = R(xr + o @ _f64(w["wo"]).T)
     hn = R(rmsnorm(h, w["g_mlp"], rms_eps))

@@ -94,6 +94,53 @@ __global__ void convert_kernel(const void* __restrict__ src, void* __restrict__ 
   }
 }
 
+// ------------------------------------------------------------------ rotary embedding
+template <int T>
+__device__ __forceinline__ float ld1(const void* base, size_t i) {
+  if (T == kF32) return reinterpret_cast<const float*>(base)[i];
+  const uint16_t v = reinterpret_cast<const uint16_t*>(base)[i];
+  return T == kF16 ? f16_lo(v) : bf16_lo(v);
+}
+template <int T>
+__device__ __forceinline__ void st1(void* base, size_t i, float x) {
+  if (T == kF32) {
+    reinterpret_cast<float*>(base)[i] = x;
+  } else {
+    reinterpret_cast<uint16_t*>(base)[i] = static_cast<uint16_t>(pack2(x, 0.f, T == kF16) & 0xFFFFu);
+  }
+}
+
+// In-place rotation of the q and k heads of qkv [T, 3*H*dh] (q | k | v column
+// blocks): pair (i, i + dh/2) of every head turns by pos * theta^(-2i/dh),
+// pos = the row's position in its segment.  One block per row at a time.
+template <int T>
+__global__ void __launch_bounds__(256) rope_kernel(void* __restrict__ qkv, const int* __restrict__ cu, int B, int T_cap,
+                                                   int H, int dh, float theta, int* err) {
+  __shared__ float2 tab[64];
+  const int half = dh / 2;
+  for (int i = threadIdx.x; i < half; i += blockDim.x) tab[i] = rope_inv_freq(i, dh, theta);
+  __syncthreads();
+  int M = cu[B];
+  if (M < 0 || M > T_cap) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) record_error(err, kErrRows);
+    M = M < 0 ? 0 : T_cap;
+  }
+  const size_t ld = static_cast<size_t>(3) * H * dh;
+  const int pairs = H * dh;                       // 2H heads (q and k) x dh/2 pairs
+  for (int row = blockIdx.x; row < M; row += gridDim.x) {
+    const float pos = static_cast<float>(row_position(cu, B, row));
+    for (int j = threadIdx.x; j < pairs; j += blockDim.x) {
+      const int hh = j / half, i = j - hh * half;
+      const size_t a = row * ld + static_cast<size_t>(hh) * dh + i, b = a + half;
+      float c, sn;
+      rope_cos_sin(pos, tab[i], c, sn);
+      const float x0 = ld1<T>(qkv, a), x1 = ld1<T>(qkv, b);
+      st1<T>(qkv, a, fmaf(x0, c, -x1 * sn));
+      st1<T>(qkv, b, fmaf(x1, c, x0 * sn));
+    }
+  }
+}
+
 // ------------------------------------------------------------------ SNR scan
 // Sec. 3.3: first 0-based i in [1, N-w] with
 //   jump  = min(s_i .. s_{i+w-1}) - s_{i-1} >= tau_jump
@@ -327,6 +374,20 @@ cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type
   SEER_CONV(kF32, kF16)
 #undef SEER_CONV
   return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_rope(void* qkv, int type, const int* cu, int B, int T_cap, int n_heads, int head_dim, float theta,
+                        int* err, int num_sms, cudaStream_t st) {
+  if (T_cap <= 0) return cudaSuccess;
+  if (head_dim % 2 != 0 || head_dim > 128) return cudaErrorInvalidValue;
+  const int blocks = T_cap < 8 * num_sms ? T_cap : 8 * num_sms;
+  switch (type) {
+    case kF32: rope_kernel<kF32><<<blocks, 256, 0, st>>>(qkv, cu, B, T_cap, n_heads, head_dim, theta, err); break;
+    case kF16: rope_kernel<kF16><<<blocks, 256, 0, st>>>(qkv, cu, B, T_cap, n_heads, head_dim, theta, err); break;
+    case kBF16: rope_kernel<kBF16><<<blocks, 256, 0, st>>>(qkv, cu, B, T_cap, n_heads, head_dim, theta, err); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
 }
 
 cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,

@@ -244,4 +244,36 @@ enum ElemType : int { kF32 = 0, kBF16 = 1, kF16 = 2 };
 
 __device__ __forceinline__ int elect_lane0() { return (threadIdx.x & 31) == 0; }
 
+// ---------------------------------------------------------------- rotary embedding
+// Inverse frequency theta^(-2i/dh) of pair i, computed in double and split into
+// a float head and tail (hi + lo equals it to ~2^-48 relative).
+__device__ __forceinline__ float2 rope_inv_freq(int i, int head_dim, float theta) {
+  const double f = exp2(-(2.0 * i / head_dim) * log2(static_cast<double>(theta)));
+  const float hi = static_cast<float>(f);
+  return make_float2(hi, static_cast<float>(f - static_cast<double>(hi)));
+}
+
+// cos and sin of pos * (f.x + f.y).  The float product pos * f.x is exact up
+// to its rounding error, which fmaf recovers; that error plus pos * f.y is a
+// small correction d (|d| < 3e-3 for pos < 2^15) applied to first order:
+// cos(a + d) = cos a - d sin a, sin(a + d) = sin a + d cos a (error d^2 / 2).
+__device__ __forceinline__ void rope_cos_sin(float pos, float2 f, float& c, float& s) {
+  const float a = __fmul_rn(pos, f.x);
+  const float d = fmaf(pos, f.y, fmaf(pos, f.x, -a));
+  float sa, ca;
+  sincosf(a, &sa, &ca);
+  c = fmaf(-d, sa, ca);
+  s = fmaf(d, ca, sa);
+}
+
+// Position of `row` inside its segment: the largest b with cu[b] <= row.
+__device__ __forceinline__ int row_position(const int* cu, int B, int row) {
+  int lo = 0, hi = B;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (cu[mid] <= row) lo = mid; else hi = mid;
+  }
+  return row - cu[lo];
+}
+
 }  // namespace seer

@@ -15,6 +15,7 @@ enum GemmMode : int {
   kGemmResidual = 1,  // C = A B^T + R
   kGemmSwiglu = 2,    // act = SiLU(A Bg^T) * (A Bu^T), optional near-zero counts
   kGemmCount = 3,     // counts only (detector): A rows gathered per sequence window
+  kGemmRope = 4,      // C = A B^T, then columns < rope_cols rotated per head (rotary embedding)
 };
 
 struct GemmParams {
@@ -37,6 +38,8 @@ struct GemmParams {
   int out_type;           // ElemType of C (kBF16 / kF16; kF32 on the CUDA-core path)
   int res_type;           // ElemType of R
   int group_m;            // raster: m-tiles per group (see tc_gemm.cu)
+  float rope_theta;       // Rope: frequency base (> 0)
+  int rope_cols;          // Rope: leading output columns that are rotated (the q|k columns)
 };
 
 struct AttnParams {
@@ -70,6 +73,8 @@ cudaError_t launch_simt_attn(const float* qkv, const AttnParams& p, cudaStream_t
 // Element-wise / scan kernels (both storage types).
 cudaError_t launch_rmsnorm(const void* x, int in_type, const void* g, void* y, int out_type, int M_cap,
                            const int* M_dev, int d, float eps, int* err, cudaStream_t st);
+cudaError_t launch_rope(void* qkv, int type, const int* cu, int B, int T_cap, int n_heads, int head_dim, float theta,
+                        int* err, int num_sms, cudaStream_t st);
 cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, cudaStream_t st);
 cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,
                             int* L_star, int* i_star, cudaStream_t st);

@@ -6,6 +6,7 @@
 
 #include <atomic>
 #include <chrono>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -207,7 +208,8 @@ seer_status check_dims(const seer_dims* dims, seer_dtype dt) {
     return fail(SEER_ERR_INVALID_ARG, "dims must be positive");
   if (d.n_heads * d.head_dim != d.d_model)
     return fail(SEER_ERR_INVALID_ARG, "n_heads * head_dim (%d) != d_model (%d)", d.n_heads * d.head_dim, d.d_model);
-  if (d.rope_theta != 0.f) return fail(SEER_ERR_UNSUPPORTED, "rotary embeddings are not implemented (rope_theta must be 0)");
+  if (!(d.rope_theta >= 0.f) || !std::isfinite(d.rope_theta))
+    return fail(SEER_ERR_INVALID_ARG, "rope_theta must be 0 (off) or a finite positive base");
   if (!(d.rms_eps >= 0.f)) return fail(SEER_ERR_INVALID_ARG, "rms_eps must be >= 0");
   if (is16(dt)) {
     if (d.d_model % 256 != 0) return fail(SEER_ERR_UNSUPPORTED, "16-bit layers need d_model %% 256 == 0 (got %d)", d.d_model);
@@ -223,8 +225,19 @@ seer_status check_dims(const seer_dims* dims, seer_dtype dt) {
 }
 
 // ------------------------------------------------------------ op launchers
+// Rotation of the q|k output columns (rotary embedding), applied by do_linear
+// when theta > 0: positions come from the segment offsets cu[0..B].
+struct RopeArgs {
+  float theta = 0.f;
+  const int32_t* cu = nullptr;
+  int B = 0;
+  int n_heads = 0;
+  int head_dim = 0;
+};
+
 seer_status do_linear(const void* a, const void* w, seer_dtype op_dt, const void* r, seer_dtype r_dt, void* c,
-                      seer_dtype c_dt, int M_cap, const int32_t* M_dev, int N, int K, cudaStream_t st, int phase) {
+                      seer_dtype c_dt, int M_cap, const int32_t* M_dev, int N, int K, cudaStream_t st, int phase,
+                      const RopeArgs& rope = RopeArgs()) {
   if (M_cap < 0 || N <= 0 || K <= 0) return fail(SEER_ERR_INVALID_ARG, "linear: bad sizes M=%d N=%d K=%d", M_cap, N, K);
   if (!a || !w || !c) return fail(SEER_ERR_INVALID_ARG, "linear: null pointer");
   if (!valid_dt(op_dt) || !valid_dt(c_dt) || (r && !valid_dt(r_dt))) return fail(SEER_ERR_INVALID_ARG, "linear: unknown dtype");
@@ -242,8 +255,18 @@ seer_status do_linear(const void* a, const void* w, seer_dtype op_dt, const void
   p.err = di->err;
   p.out_type = c_dt;
   p.res_type = r ? r_dt : c_dt;
-  const int mode = r ? kGemmResidual : kGemmStore;
+  const bool rot = rope.theta > 0.f;
+  if (rot && (r || !rope.cu || rope.B <= 0 || N != 3 * rope.n_heads * rope.head_dim))
+    return fail(SEER_ERR_INVALID_ARG, "linear: the rotary epilogue needs a q|k|v output, cu_seqlens and no residual");
+  const int mode = r ? kGemmResidual : (rot ? kGemmRope : kGemmStore);
+  if (rot) {
+    p.rope_theta = rope.theta;
+    p.rope_cols = 2 * rope.n_heads * rope.head_dim;
+    p.cu = rope.cu;
+    p.B = rope.B;
+  }
   if (is16(op_dt)) {
+    if (rot && rope.head_dim != 128) return fail(SEER_ERR_UNSUPPORTED, "16-bit rotary epilogue needs head_dim == 128");
     if (!is16(c_dt) || (r && !is16(r_dt))) return fail(SEER_ERR_UNSUPPORTED, "16-bit linear needs 16-bit output and residual");
     if (N % 256 != 0 || K % 64 != 0)
       return fail(SEER_ERR_UNSUPPORTED, "16-bit linear needs N %% 256 == 0 and K %% 64 == 0 (N=%d K=%d)", N, K);
@@ -261,8 +284,13 @@ seer_status do_linear(const void* a, const void* w, seer_dtype op_dt, const void
     if (c_dt != SEER_F32 || (r && r_dt != SEER_F32)) return fail(SEER_ERR_UNSUPPORTED, "fp32 linear needs fp32 output");
     if (M_cap == 0) return SEER_OK;
     Phase ph(phase, st);
-    SEER_CUDA(launch_simt_gemm(mode, static_cast<const float*>(a), static_cast<const float*>(w), nullptr, p, st),
+    SEER_CUDA(launch_simt_gemm(rot ? kGemmStore : mode, static_cast<const float*>(a), static_cast<const float*>(w),
+                               nullptr, p, st),
               "simt_gemm launch");
+    if (rot)
+      SEER_CUDA(launch_rope(c, kF32, rope.cu, rope.B, M_cap, rope.n_heads, rope.head_dim, rope.theta, di->err,
+                            di->num_sms, st),
+                "rope launch");
   }
   return SEER_OK;
 }
@@ -478,6 +506,22 @@ seer_status seer_linear(const void* a, const void* w, seer_dtype op_dt, const vo
                    r ? PH_OPROJ : PH_QKV);
 }
 
+seer_status seer_rope(void* qkv, seer_dtype dt, const int32_t* cu_seqlens, int B, int T_capacity, int n_heads,
+                      int head_dim, float theta, void* stream) {
+  if (!valid_dt(dt)) return fail(SEER_ERR_INVALID_ARG, "rope: unknown dtype");
+  if (!qkv || !cu_seqlens) return fail(SEER_ERR_INVALID_ARG, "rope: null pointer");
+  if (B <= 0 || T_capacity < 0 || n_heads <= 0 || head_dim <= 0) return fail(SEER_ERR_INVALID_ARG, "rope: bad sizes");
+  if (!(theta > 0.f) || !std::isfinite(theta)) return fail(SEER_ERR_INVALID_ARG, "rope: theta must be finite and > 0");
+  if (head_dim % 2 != 0 || head_dim > 128) return fail(SEER_ERR_UNSUPPORTED, "rope: head_dim must be even and <= 128");
+  DeviceInfo* di;
+  SEER_TRY(device_info(&di));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Phase ph(PH_QKV, st);
+  SEER_CUDA(launch_rope(qkv, dt, cu_seqlens, B, T_capacity, n_heads, head_dim, theta, di->err, di->num_sms, st),
+            "rope launch");
+  return SEER_OK;
+}
+
 seer_status seer_swiglu(const void* a, const void* w_gate, const void* w_up, seer_dtype op_dt, void* act,
                         seer_dtype act_dt, int M_cap, const int32_t* M_dev, int F, int K, const int32_t* cu_seqlens,
                         int B, const int32_t* count_resp_start, int N, float act_eps, int32_t* counts_out,
@@ -610,7 +654,13 @@ seer_status seer_layer_forward(const seer_layer_weights* w, const seer_dims* dim
   const float eps = dims->rms_eps;
 
   SEER_TRY(do_rmsnorm(x, dt, w->g_attn, xn, it, T_capacity, M_dev, d, eps, st, PH_NORM1));
-  SEER_TRY(do_linear(xn, w->w_qkv, it, nullptr, it, qkv, it, T_capacity, M_dev, 3 * d, d, st, PH_QKV));
+  RopeArgs rope;
+  rope.theta = dims->rope_theta;
+  rope.cu = cu_seqlens;
+  rope.B = B;
+  rope.n_heads = H;
+  rope.head_dim = dh;
+  SEER_TRY(do_linear(xn, w->w_qkv, it, nullptr, it, qkv, it, T_capacity, M_dev, 3 * d, d, st, PH_QKV, rope));
   SEER_TRY(do_attention(qkv, xn, it, cu_seqlens, kv_len, B, T_capacity, H, dh, sched, L.total - L.off_sched, st));
   SEER_TRY(do_linear(xn, w->w_o, it, x, dt, h, it, T_capacity, M_dev, d, d, st, PH_OPROJ));
   SEER_TRY(do_rmsnorm(h, it, w->g_mlp, xn, it, T_capacity, M_dev, d, eps, st, PH_NORM2));

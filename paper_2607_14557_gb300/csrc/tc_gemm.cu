@@ -20,6 +20,8 @@
 //   Swiglu    B = [Wg tile ; Wu tile] -> act = SiLU(g) * u  (gate/up), plus the
 //             per-row count of |act| < eps on response rows (step-0 hook)
 //   Count     detector: A rows gathered per sequence window, counts only
+//   Rope      Store, then the q|k columns rotated per 128-wide head by the
+//             rotary embedding at each row's position in its sequence
 #include "common.cuh"
 #include "kernels.h"
 
@@ -37,7 +39,9 @@ constexpr int THREADS = 192;
 constexpr int ACC_COLS = 256;
 constexpr int TMEM_COLS = 512;
 constexpr int BAR_BYTES = 256;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
+constexpr int ROPE_HEAD = 128;                       // head width of the Rope epilogue
+constexpr int ROPE_BYTES = ROPE_HEAD / 2 * 8;        // (hi, lo) inverse frequency per pair
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + ROPE_BYTES + 1024;
 
 // Raster: groups of `group_m` m-tiles; inside a group m varies fastest and
 // the group sweeps every n-tile.  group_m = 1 keeps the whole B operand hot in
@@ -67,6 +71,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint64_t* acc_empty = acc_full + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float2* rope_tab = reinterpret_cast<float2*>(smem + STAGES * STAGE_BYTES + BAR_BYTES);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -194,6 +199,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int q = warp & 3;                    // TMEM lane quarter owned by this warp
     const int row_in_tile = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    if (MODE == kGemmRope) {
+      const int et = threadIdx.x - 64;                 // 0..127 over the epilogue warps
+      if (et < ROPE_HEAD / 2) rope_tab[et] = rope_inv_freq(et, ROPE_HEAD, p.rope_theta);
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+    }
     int acc = 0;
     uint32_t acc_ph = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
@@ -202,7 +212,50 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!mbar_wait(&acc_full[acc], acc_ph, abort_flag, p.err)) break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + lane_off + static_cast<uint32_t>(acc * ACC_COLS);
-      if (MODE == kGemmStore || MODE == kGemmResidual) {
+      if (MODE == kGemmRope) {
+        // the tile holds two heads; pair (c, c + 64) of a head rotates by pos * f_c
+        const int row = m * BM + row_in_tile;
+        const bool valid = row < M;
+        const bool rotate = n * BN < p.rope_cols;       // tile-uniform (rope_cols % BN == 0)
+        const bool of16 = p.out_type == kF16;
+        uint16_t* crow = reinterpret_cast<uint16_t*>(p.C) + static_cast<size_t>(valid ? row : 0) * p.ldc + n * BN;
+        const float pos = (valid && rotate) ? static_cast<float>(row_position(p.cu, p.B, row)) : 0.f;
+#pragma unroll 1
+        for (int c = 0; c < ROPE_HEAD / 64; ++c) {
+          float cs[32], sn[32];
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            if (rotate) rope_cos_sin(pos, rope_tab[c * 32 + e], cs[e], sn[e]);
+            else { cs[e] = 1.f; sn[e] = 0.f; }
+          }
+#pragma unroll 1
+          for (int hh = 0; hh < BN / ROPE_HEAD; ++hh) {
+            const int c0 = hh * ROPE_HEAD + c * 32, c1 = c0 + ROPE_HEAD / 2;
+            uint32_t r0[32], r1[32];
+            tmem_ld32(tacc + c0, r0);
+            tmem_ld32(tacc + c1, r1);
+            tmem_ld_wait();
+            if (valid) {
+              float v0[32], v1[32];
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                const float x0 = __uint_as_float(r0[e]), x1 = __uint_as_float(r1[e]);
+                v0[e] = fmaf(x0, cs[e], -x1 * sn[e]);
+                v1[e] = fmaf(x1, cs[e], x0 * sn[e]);
+              }
+              uint4* p0 = reinterpret_cast<uint4*>(crow + c0);
+              uint4* p1 = reinterpret_cast<uint4*>(crow + c1);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                p0[i] = make_uint4(pack2(v0[8 * i + 0], v0[8 * i + 1], of16), pack2(v0[8 * i + 2], v0[8 * i + 3], of16),
+                                   pack2(v0[8 * i + 4], v0[8 * i + 5], of16), pack2(v0[8 * i + 6], v0[8 * i + 7], of16));
+                p1[i] = make_uint4(pack2(v1[8 * i + 0], v1[8 * i + 1], of16), pack2(v1[8 * i + 2], v1[8 * i + 3], of16),
+                                   pack2(v1[8 * i + 4], v1[8 * i + 5], of16), pack2(v1[8 * i + 6], v1[8 * i + 7], of16));
+              }
+            }
+          }
+        }
+      } else if (MODE == kGemmStore || MODE == kGemmResidual) {
         const int row = m * BM + row_in_tile;
         const bool valid = row < M;
         const bool of16 = p.out_type == kF16, rf16 = p.res_type == kF16;
@@ -335,6 +388,7 @@ cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& m
     case kGemmResidual: return launch_mode<kGemmResidual>(mA, mB0, mB1, p, num_sms, st);
     case kGemmSwiglu: return launch_mode<kGemmSwiglu>(mA, mB0, mB1, p, num_sms, st);
     case kGemmCount: return launch_mode<kGemmCount>(mA, mB0, mB1, p, num_sms, st);
+    case kGemmRope: return launch_mode<kGemmRope>(mA, mB0, mB1, p, num_sms, st);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -75,6 +75,7 @@ def lib() -> ctypes.CDLL:
             "seer_layer_workspace_size": [ctypes.POINTER(seer_dims), i32, i32, i32, ctypes.POINTER(sz)],
             "seer_rmsnorm": [vp, i32, vp, vp, i32, i32, vp, i32, ctypes.c_float, vp],
             "seer_linear": [vp, vp, i32, vp, i32, vp, i32, i32, vp, i32, i32, vp],
+            "seer_rope": [vp, i32, vp, i32, i32, i32, i32, ctypes.c_float, vp],
             "seer_swiglu": [vp, vp, vp, i32, vp, i32, i32, vp, i32, i32, vp, i32, vp, i32, ctypes.c_float, vp, vp],
             "seer_convert": [vp, i32, vp, i32, sz, vp],
             "seer_attention": [vp, vp, i32, vp, vp, i32, i32, i32, i32, vp, sz, vp],
@@ -185,6 +186,10 @@ def seer_rmsnorm(x, x_dt, g, y, y_dt, M_cap, M_dev, d, eps, stream=None):
 def seer_linear(a, w, op_dt, r, r_dt, c, c_dt, M_cap, M_dev, N, K, stream=None):
     _check(lib().seer_linear(_p(a), _p(w), _dt(op_dt), _p(r), _dt(r_dt), _p(c), _dt(c_dt), M_cap, _p(M_dev), N, K,
                              _stream(stream)))
+
+
+def seer_rope(qkv, dt, cu_seqlens, B, T_capacity, n_heads, head_dim, theta, stream=None):
+    _check(lib().seer_rope(_p(qkv), _dt(dt), _p(cu_seqlens), B, T_capacity, n_heads, head_dim, theta, _stream(stream)))
 
 
 def seer_swiglu(a, w_gate, w_up, op_dt, act, act_dt, M_cap, M_dev, F, K, cu_seqlens=None, B=0, count_resp_start=None,

@@ -43,8 +43,12 @@ def test_host_side_argument_checks_need_no_gpu(libseer):
     assert out.value > 1000 * 4096 * 2 * 6
     assert L.seer_layer_workspace_size(ctypes.byref(bad), S.SEER_BF16, 1000, 4, ctypes.byref(out)) == 1
     rope = S.make_dims(4096, 32, 128, 12288, rope_theta=10000.0)
-    assert L.seer_layer_workspace_size(ctypes.byref(rope), S.SEER_BF16, 1000, 4, ctypes.byref(out)) == 2
+    assert L.seer_layer_workspace_size(ctypes.byref(rope), S.SEER_BF16, 1000, 4, ctypes.byref(out)) == 0
+    neg = S.make_dims(4096, 32, 128, 12288, rope_theta=-1.0)
+    assert L.seer_layer_workspace_size(ctypes.byref(neg), S.SEER_BF16, 1000, 4, ctypes.byref(out)) == 1
     assert b"rope" in L.seer_last_error()
+    nan = S.make_dims(4096, 32, 128, 12288, rope_theta=float("nan"))
+    assert L.seer_layer_workspace_size(ctypes.byref(nan), S.SEER_BF16, 1000, 4, ctypes.byref(out)) == 1
 
 
 def test_poll_ctrl_times_out_on_host_flag_never_set(libseer):

@@ -21,14 +21,14 @@ def _device_clean():
     assert S.seer_check_device() == 0
 
 
-def run_path(wl, lens=None, tau_pad=0.2, extra_cap=64, data=None):
+def run_path(wl, lens=None, tau_pad=0.2, extra_cap=64, data=None, rope_theta=0.0):
     """Detect, pack and run one layer on the GPU; return everything needed to check it."""
     dt = wl.dtype
     lens = lens or synth.lengths(wl)
     x, cu_full, resp = data if data is not None else synth.hidden_full(wl, lens)
     w = synth.layer_weights(wl, 0)
     B, N, F, d = wl.batch, wl.window, wl.d_ff, wl.d
-    dims = S.make_dims(d, wl.n_heads, wl.head_dim, F)
+    dims = S.make_dims(d, wl.n_heads, wl.head_dim, F, rope_theta=rope_theta)
     params = S.make_params(wl.act_eps, tau_pad=tau_pad)
     W, WL = layer_weight_tensors(wl, w)
     xd = to_dev(x, dt)
@@ -47,7 +47,8 @@ def run_path(wl, lens=None, tau_pad=0.2, extra_cap=64, data=None):
     S.seer_layer_forward(weights_struct(WL), dims, dt, xp, y, cu, kv, B, T_cap, None, 0, 0.0, None, ws, ws_bytes)
     torch.cuda.synchronize()
     return dict(x=x, cu_full=cu_full, resp=resp, w=w, lens=lens, counts=counts.cpu().numpy().reshape(B, N),
-                L=L.cpu().numpy(), cu=cu.cpu().numpy(), kv=kv.cpu().numpy(), xp=host(xp), y=host(y), T_cap=T_cap)
+                L=L.cpu().numpy(), cu=cu.cpu().numpy(), kv=kv.cpu().numpy(), xp=host(xp), y=host(y), T_cap=T_cap,
+                rope_theta=rope_theta)
 
 
 def _check_path(wl, r):
@@ -58,7 +59,7 @@ def _check_path(wl, r):
     np.testing.assert_array_equal(r["kv"], kv)
     T = int(cu[-1])
     np.testing.assert_array_equal(r["xp"][:T], oracle.pack_rows(r["x"], r["cu_full"], seg))
-    ref = oracle.layer_forward_packed(r["xp"][:T], cu, r["w"], wl.n_heads, kv_len=kv)
+    ref = oracle.layer_forward_packed(r["xp"][:T], cu, r["w"], wl.n_heads, kv_len=kv, rope_theta=r["rope_theta"])
     err = check_close(r["y"][:T], ref, wl.dtype, wl.name)
     assert (r["y"][T:] == 9.0).all()                                    # zero work past truncation
     return err
@@ -169,3 +170,43 @@ def test_naive_pad_comparator_matches_truncated_rows():
         n = int(lens.ctx[b] + L[b])
         np.testing.assert_array_equal(ynh[cun_h[b]:cun_h[b] + n], yt[cu_t[b]:cu_t[b] + n])
     assert np.isfinite(ynh).all()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_path_with_rotary_embedding(dtype):
+    # optional rotary q/k embedding: fused into the QKV epilogue (16-bit) or a separate kernel (fp32)
+    if dtype == "bf16":
+        wl = synth.tiny_workload(dtype="bf16", seed=350, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4,
+                                 window=200, boundary=("uniform", 8, 190), visual=("mult", 96, 1, 3))
+    else:
+        wl = synth.workload(0)
+    r = run_path(wl, rope_theta=1e4)
+    _check_path(wl, r)
+
+
+def test_rotary_layer_at_long_positions():
+    # one 9k-row segment: rotation angles up to ~9000 rad in the fused epilogue (sampled query rows)
+    wl = synth.tiny_workload(dtype="bf16", seed=360, d=256, n_heads=2, head_dim=128, d_ff=768, batch=2,
+                             window=128, visual=("mult", 4000, 2, 2), prompt=("uniform", 900, 990),
+                             boundary=("uniform", 20, 100))
+    lens = synth.lengths(wl)
+    x, cu_full, _ = synth.hidden_full(wl, lens)
+    w = synth.layer_weights(wl, 0)
+    d, F, B = wl.d, wl.d_ff, wl.batch
+    dims = S.make_dims(d, wl.n_heads, wl.head_dim, F, rope_theta=1e4)
+    W, WL = layer_weight_tensors(wl, w)
+    T = x.shape[0]
+    y = torch.empty((T, d), dtype=torch.bfloat16, device=cuda())
+    ws_bytes = S.seer_layer_workspace_size(dims, "bf16", T, B)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=cuda())
+    S.seer_layer_forward(weights_struct(WL), dims, "bf16", to_dev(x, "bf16"), y, i32(cu_full), None, B, T, None, 0,
+                         0.0, None, ws, ws_bytes)
+    torch.cuda.synchronize()
+    yh = host(y)
+    rng = np.random.default_rng(3)
+    for b in range(B):
+        L = int(cu_full[b + 1] - cu_full[b])
+        assert L > 8000
+        rows = sorted({0, 1, L - 1, L - 2, *map(int, rng.integers(L // 2, L, 14))})
+        ref = oracle.layer_forward_rows(x[cu_full[b]:cu_full[b + 1]], w, wl.n_heads, rows, rope_theta=1e4)
+        check_close(yh[cu_full[b] + np.asarray(rows)], ref, "bf16", f"rotary layer segment {b}")
