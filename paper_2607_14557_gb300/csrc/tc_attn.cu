@@ -5,26 +5,28 @@
 // the first kv_len[b] rows of the same segment, with no causal mask; rows
 // beyond kv_len (bucket padding of the static path) are never keys.
 //
-// One CTA per (segment, head, 128-query tile); 64 + 128 * NGRP threads:
-//   warp 0     TMA producers: Q once, then K_j (lane 0) and V_j (lane 1),
-//              128 keys x 128 dims with 128-byte swizzle, each in a 3-deep
-//              ring (key tiles take ~2000 cycles to land under load);
-//   warp 1     TMEM allocator + MMA issuer: S_j = Q K_j^T (M=N=128, K=16 x 8)
-//              into one of two S buffers, then O += P_j V_j (V as an MN-major
-//              operand) into the O accumulator.  Q and P are A operands read
-//              from tensor memory, so each MMA streams only its B operand
-//              from shared memory (shared-memory bandwidth bounds an
-//              all-shared-memory version);
-//   warps 2.. softmax, NGRP groups of four warps: a query row (one TMEM
-//              lane) is shared by one thread of each group, which owns
-//              128 / NGRP of the key columns (and of the output dims); the
-//              parts of a row exchange their maxima through shared memory
-//              once per key tile (an mbarrier, so every wait is bounded).
-//              Online softmax in the log2 domain with lazy rescaling: O is
-//              rescaled in TMEM only when the running max grows by more than
-//              2^8.  The softmax warps stage Q into tensor memory once and
-//              write each P_j there (tcgen05.st).
-// The QK^T MMAs run up to two key tiles ahead of the softmax.
+// One CTA per (segment, head, pair of 128-query tiles); 384 threads:
+//   warp 0     TMA producers: both Q tiles once, then K_j (lane 0, 3-deep
+//              ring) and V_j (lane 1, 2-deep ring), 128 keys x 128 dims with
+//              128-byte swizzle;
+//   warps 1-2  TMEM allocator (warp 1) and one MMA issuer per query tile t:
+//              O_t += P_t,j-1 V_j-1 (P from tensor memory, V an MN-major
+//              shared operand), then S_t,j = Q_t K_j^T (both from shared
+//              memory).  The tensor pipe executes one thread's MMAs in issue
+//              order, so S_t,j may overwrite the columns that held P_t,j-1.
+//              Two issuers keep one tile's barrier waits off the other
+//              tile's MMA stream (the pipe's issue queue is shallow); a turn
+//              token passed between them keeps the rounds in ping-pong order
+//              (tile 0's PV + QK^T, then tile 1's), so the two softmax groups
+//              work in alternation instead of in lock step;
+//   warps 4-7  softmax of query tile 0, warps 8-11 of tile 1: one thread per
+//              query row holds the row's 128 scores, so no exchange between
+//              threads is needed.  While one group exponentiates its tile,
+//              the tensor pipe multiplies the other tile (ping-pong).
+// Online softmax in the log2 domain with lazy rescaling: O_t is rescaled in
+// tensor memory only when the running max grows by more than 2^8.
+// Tensor memory (512 columns): S_0 | S_1 | O_0 | O_1, P_t packed into the
+// first 64 columns of S_t.
 // The schedule kernel orders work units longest segment first.
 #include <math.h>
 
@@ -37,26 +39,21 @@ namespace {
 constexpr int BQ = 128;
 constexpr int BKV = 128;
 constexpr int DH = 128;
-constexpr int NGRP = 2;                     // softmax column groups (4 warps each)
-constexpr int COLS = BKV / NGRP;            // key columns / output dims per softmax thread
-constexpr int SOFTMAX_WARPS = 4 * NGRP;
-constexpr int THREADS = 64 + 32 * SOFTMAX_WARPS;
-constexpr int TILE_BYTES = 128 * DH * 2;   // 32 KB: 128 rows x 128 16-bit values as two 16 KB swizzle panels
+constexpr int NT = 2;                       // query tiles per CTA
+constexpr int THREADS = 128 + 128 * NT;    // warps 0-3 producer/issuers, 4 warps per tile
+constexpr int TILE_BYTES = 128 * DH * 2;    // 32 KB: 128 rows x 128 16-bit values as two 16 KB swizzle panels
 constexpr int PANEL = 16384;
-// Six 32 KB slots: Q in slot 0 (free again once Q sits in tensor memory),
-// K stages 0, 1, 2 in slots 1, 2, 0 and V stages 0, 1, 2 in slots 3, 4, 5.
-constexpr int KV_STAGES = 3;
-constexpr int OFF_Q = 0;
-__host__ __device__ constexpr int k_slot(int st) { return (st == 2 ? 0 : st + 1) * TILE_BYTES; }
-__host__ __device__ constexpr int v_slot(int st) { return (3 + st) * TILE_BYTES; }
-constexpr int OFF_BAR = 6 * TILE_BYTES;
-constexpr int OFF_RED = OFF_BAR + 256;      // float max[2 tiles][NGRP][128] + float sum[NGRP][128]
-constexpr int SMEM_BYTES = OFF_RED + (2 * NGRP * 128 + NGRP * 128) * 4 + 1024;
+constexpr int K_STAGES = 3;
+constexpr int V_STAGES = 2;
+constexpr int OFF_Q = 0;                                   // Q tiles 0, 1
+constexpr int OFF_K = NT * TILE_BYTES;
+constexpr int OFF_V = OFF_K + K_STAGES * TILE_BYTES;
+constexpr int OFF_BAR = OFF_V + V_STAGES * TILE_BYTES;
+constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+static_assert(SMEM_BYTES <= 232448, "shared memory per CTA");
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t TM_O = 256;              // TMEM columns: S0 [0,128), S1 [128,256), O [256,384),
-constexpr uint32_t TM_Q = 384;              //   Q [384,448) and P [448,512) as packed 16-bit pairs
-constexpr uint32_t TM_P = 448;
-static_assert(NGRP == 2, "the TMEM staging of Q and P assumes two 64-column groups");
+constexpr uint32_t TM_S = 0;                // S_t at TM_S + 128 t
+constexpr uint32_t TM_O = 256;              // O_t at TM_O + 128 t
 constexpr float RESCALE_THRESHOLD = 8.0f;   // log2 units
 
 __device__ __forceinline__ float ex2(float x) {
@@ -65,17 +62,66 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float y;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+  return y;
+}
+
+// 2^x of two packed f16 values in one MUFU operation.
+__device__ __forceinline__ uint32_t ex2_h2(uint32_t x) {
+  uint32_t y;
+  asm("ex2.approx.f16x2 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+// acc + (f16 half of v), in fp32 (mixed-precision add).
+__device__ __forceinline__ float add_f16_lo(uint32_t v, float acc) {
+  float d;
+  asm("{\n\t.reg .b16 l, h;\n\tmov.b32 {l, h}, %1;\n\tadd.rn.f32.f16 %0, l, %2;\n\t}" : "=f"(d) : "r"(v), "f"(acc));
+  return d;
+}
+__device__ __forceinline__ float add_f16_hi(uint32_t v, float acc) {
+  float d;
+  asm("{\n\t.reg .b16 l, h;\n\tmov.b32 {l, h}, %1;\n\tadd.rn.f32.f16 %0, h, %2;\n\t}" : "=f"(d) : "r"(v), "f"(acc));
+  return d;
+}
+
+// Packed probabilities of keys 32c .. 32c+31 of one row: p = 2^(s * scale - m),
+// accumulated into the row sum.  f16: the exponent x is rounded to f16 and
+// two probabilities come from one MUFU operation (ex2.approx.f16x2) -- the
+// MUFU unit, not the tensor pipe, otherwise bounds a row's softmax; P is
+// stored in f16 anyway.  bf16: one fp32 ex2 per probability.
+template <bool F16>
+__device__ __forceinline__ void row_probs(const float* s, float scale_log2, float neg, float (&rs)[4],
+                                          uint32_t (&pk)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const float x0 = fmaf(s[2 * i], scale_log2, neg);
+    const float x1 = fmaf(s[2 * i + 1], scale_log2, neg);
+    if (F16) {
+      const uint32_t ph = ex2_h2(pack_f16x2(x0, x1));
+      rs[(2 * i) & 3] = add_f16_lo(ph, rs[(2 * i) & 3]);
+      rs[(2 * i + 1) & 3] = add_f16_hi(ph, rs[(2 * i + 1) & 3]);
+      pk[i] = ph;
+    } else {
+      const float p0 = ex2(x0), p1 = ex2(x1);
+      rs[i & 3] += p0 + p1;
+      pk[i] = pack_bf16x2(p0, p1);
+    }
+  }
+}
+
 template <bool F16>
 __global__ void __launch_bounds__(THREADS, 1)
     tc_attn_kernel(const __grid_constant__ CUtensorMap mQKV, const AttnParams p) {
   const int u = blockIdx.x;
   if (u >= *p.work_count) return;
   const int4 wk = p.work[u];
-  const int b = wk.x, h = wk.y, qt = wk.z;
+  const int b = wk.x, h = wk.y, qt0 = wk.z, nt = wk.w;   // query tiles qt0 .. qt0 + nt - 1
   const int seq0 = p.cu[b];
   const int L = p.cu[b + 1] - seq0;
   const int kvL = p.kv_len ? p.kv_len[b] : L;
-  const int q0 = seq0 + qt * BQ;
+  const int q0 = seq0 + qt0 * BQ;
   const int nkv = (kvL + BKV - 1) / BKV;
   const int D = p.n_heads * DH;
   const int xq = h * DH, xk = D + h * DH, xv = 2 * D + h * DH;
@@ -84,42 +130,36 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;     // [KV_STAGES]
-  uint64_t* k_empty = bars + 4;    // [KV_STAGES]
-  uint64_t* v_full = bars + 7;     // [KV_STAGES]
-  uint64_t* v_empty = bars + 10;   // [KV_STAGES]
-  uint64_t* s_full = bars + 13;    // [2]
-  uint64_t* s_empty = bars + 15;   // [2]
-  uint64_t* p_full = bars + 17;
-  uint64_t* pv_done = bars + 18;
-  uint64_t* max_ready = bars + 19; // [2] row-max exchange, one per tile parity
-  uint64_t* sum_ready = bars + 21;
-  uint64_t* q_staged = bars + 22;  // Q copied from shared to tensor memory
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 23);
+  uint64_t* k_full = bars + 1;               // [K_STAGES]
+  uint64_t* k_empty = k_full + K_STAGES;     // [K_STAGES]
+  uint64_t* v_full = k_empty + K_STAGES;     // [V_STAGES]
+  uint64_t* v_empty = v_full + V_STAGES;     // [V_STAGES]
+  uint64_t* s_full = v_empty + V_STAGES;     // [NT] S_t,j written (and O_t += P_t,j-1 V done)
+  uint64_t* p_full = s_full + NT;            // [NT] P_t,j in tensor memory (O_t rescaled)
+  uint64_t* o_done = p_full + NT;            // [NT] last PV of tile t complete
+  uint64_t* turn = o_done + NT;              // [NT] issuer t may enqueue its next round
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(turn + NT);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* red_max = reinterpret_cast<float*>(smem + OFF_RED);   // [2 tiles][NGRP][128] partial row maxima
-  float* red_sum = red_max + 2 * NGRP * 128;                   // [NGRP][128] partial row sums
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int i = 0; i < KV_STAGES; ++i) {
+    for (int i = 0; i < K_STAGES; ++i) {
       mbar_init(&k_full[i], 1);
-      mbar_init(&k_empty[i], 1);
+      mbar_init(&k_empty[i], nt);      // one commit per tile issuer
+    }
+    for (int i = 0; i < V_STAGES; ++i) {
       mbar_init(&v_full[i], 1);
-      mbar_init(&v_empty[i], 1);
+      mbar_init(&v_empty[i], nt);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&s_full[i], 1);
-      mbar_init(&s_empty[i], SOFTMAX_WARPS);
-      mbar_init(&max_ready[i], SOFTMAX_WARPS);
+    for (int t = 0; t < NT; ++t) {
+      mbar_init(&s_full[t], 1);
+      mbar_init(&p_full[t], 4);
+      mbar_init(&o_done[t], 1);
+      mbar_init(&turn[t], 1);
     }
-    mbar_init(p_full, SOFTMAX_WARPS);
-    mbar_init(pv_done, 1);
-    mbar_init(sum_ready, SOFTMAX_WARPS);
-    mbar_init(q_staged, SOFTMAX_WARPS);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -135,22 +175,23 @@ __global__ void __launch_bounds__(THREADS, 1)
     // buffer (freed by PV) never delays the next K (needed by QK^T).
     if (lane == 0) {
       tma_prefetch_desc(&mQKV);
-      mbar_arrive_expect_tx(q_full, TILE_BYTES);
-      tma_load_2d(smem + OFF_Q, &mQKV, q_full, xq, q0);
-      tma_load_2d(smem + OFF_Q + PANEL, &mQKV, q_full, xq + 64, q0);
+      mbar_arrive_expect_tx(q_full, nt * TILE_BYTES);
+      for (int t = 0; t < nt; ++t) {
+        tma_load_2d(smem + OFF_Q + t * TILE_BYTES, &mQKV, q_full, xq, q0 + t * BQ);
+        tma_load_2d(smem + OFF_Q + t * TILE_BYTES + PANEL, &mQKV, q_full, xq + 64, q0 + t * BQ);
+      }
     }
     if (lane < 2) {
       const bool is_k = lane == 0;
+      const int stages = is_k ? K_STAGES : V_STAGES;
       uint64_t* full = is_k ? k_full : v_full;
       uint64_t* empty = is_k ? k_empty : v_empty;
       const int x = is_k ? xk : xv;
       int issued = 0;
       for (int j = 0; j < nkv; ++j) {
-        const int st = j % KV_STAGES, use = j / KV_STAGES;
+        const int st = j % stages, use = j / stages;
         if (use > 0 && !mbar_wait(&empty[st], (use - 1) & 1, abort_flag, p.err)) break;
-        // K stage 2 reuses Q's slot: wait until Q has been staged in tensor memory
-        if (is_k && j == 2 && !mbar_wait(q_staged, 0, abort_flag, p.err)) break;
-        uint8_t* dst = smem + (is_k ? k_slot(st) : v_slot(st));
+        uint8_t* dst = smem + (is_k ? OFF_K : OFF_V) + st * TILE_BYTES;
         mbar_arrive_expect_tx(&full[st], TILE_BYTES);
         tma_load_2d(dst, &mQKV, &full[st], x, seq0 + j * BKV);
         tma_load_2d(dst + PANEL, &mQKV, &full[st], x + 64, seq0 + j * BKV);
@@ -158,228 +199,169 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       if (*abort_flag) {
         if (is_k) mbar_wait_drain(q_full, 0, 200000000ull);
-        for (int j = issued > KV_STAGES ? issued - KV_STAGES : 0; j < issued; ++j)
-          mbar_wait_drain(&full[j % KV_STAGES], (j / KV_STAGES) & 1, 200000000ull);
+        for (int j = issued > stages ? issued - stages : 0; j < issued; ++j)
+          mbar_wait_drain(&full[j % stages], (j / stages) & 1, 200000000ull);
       }
     }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
-      // Issues QK^T for tile js as soon as K_js has landed and its S buffer is
-      // free (up to two tiles ahead of the softmax), and PV for tile jp as soon
-      // as P_jp is ready; both conditions are polled, never blocked on, so a
-      // slow softmax never holds back the next QK^T.
+  } else if (warp == 1 || warp == 2) {
+    const int t = warp - 1;
+    if (lane == 0 && t < nt) {
+      // ------------------------------------------------ MMA issuer of tile t
       constexpr uint32_t idesc_qk = make_idesc(BQ, BKV, 0, F16);
       constexpr uint32_t idesc_pv = make_idesc(BQ, DH, 1, F16);
-      bool ok = mbar_wait(q_staged, 0, abort_flag, p.err);
-      int js = 0, jp = 0;
-      uint64_t t_idle = 0;
-      uint32_t spins = 0;
-      while (ok && jp < nkv) {
-        bool progressed = false;
-        if (js < nkv) {
-          const int sb = js & 1, use = js >> 1;
-          const int kst = js % KV_STAGES, kuse = js / KV_STAGES;
-          if (mbar_test_wait(&k_full[kst], kuse & 1) && (use == 0 || mbar_test_wait(&s_empty[sb], (use - 1) & 1))) {
-            tc_fence_after();
-            const uint32_t sk = smem_u32(smem + k_slot(kst));
+      // descriptors built once; a K=16 step adds a constant to the
+      // start-address field (stage s of a ring: + s * TILE_BYTES / 16)
+      const uint64_t dq = make_sdesc_sw128(smem_u32(smem + OFF_Q + t * TILE_BYTES), 16, 1024);
+      const uint64_t dk0 = make_sdesc_sw128(smem_u32(smem + OFF_K), 16, 1024);
+      const uint64_t dv0 = make_sdesc_sw128(smem_u32(smem + OFF_V), PANEL, 1024);
+      const uint32_t dS = tmem + TM_S + 128 * t, dO = tmem + TM_O + 128 * t;
+      bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
+      for (int j = 0; ok && j <= nkv; ++j) {
+        // everything this round needs, then the turn: round j of tile 1
+        // follows round j of tile 0, which follows round j-1 of tile 1
+        const int jv = j - 1, vs = jv % V_STAGES, ks = j % K_STAGES;
+        if ((j > 0 && (!mbar_wait(&v_full[vs], (jv / V_STAGES) & 1, abort_flag, p.err) ||
+                       !mbar_wait(&p_full[t], jv & 1, abort_flag, p.err))) ||
+            (j < nkv && !mbar_wait(&k_full[ks], (j / K_STAGES) & 1, abort_flag, p.err))) {
+          ok = false;
+          break;
+        }
+        if (nt > 1 && (t == 1 || j > 0) && !mbar_wait(&turn[t], (t == 1 ? j : j - 1) & 1, abort_flag, p.err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (j > 0) {
+          // O_t += P_t,j-1 V_j-1: A = P from tensor memory (8 columns per 16
+          // keys); B = V [keys, dims] with dims contiguous, an MN-major
+          // operand whose two 64-dim panels are PANEL bytes apart (LBO) and
+          // 8-key groups 1 KB apart (SBO)
 #pragma unroll
-            for (int k = 0; k < DH / 16; ++k) {
-              // A = Q from tensor memory, B = K_js (K-major, 128-byte swizzle)
-              const uint32_t off = (k >> 2) * PANEL + (k & 3) * 32;
-              tc_mma_f16_tmem_a(tmem + sb * 128, tmem + TM_Q + 8 * k, make_sdesc_sw128(sk + off, 16, 1024), idesc_qk,
-                                k > 0 ? 1u : 0u);
-            }
-            tc_commit(&k_empty[kst]);
-            tc_commit(&s_full[sb]);
-            ++js;
-            progressed = true;
-          }
+          for (int k = 0; k < BKV / 16; ++k)
+            tc_mma_f16_tmem_a(dO, dS + 8 * k, dv0 + static_cast<uint64_t>(vs * (TILE_BYTES >> 4) + k * 128), idesc_pv,
+                              (jv > 0 || k > 0) ? 1u : 0u);
+          tc_commit(&v_empty[vs]);
+          if (j == nkv) tc_commit(&o_done[t]);
         }
-        if (jp < js) {
-          const int vst = jp % KV_STAGES, vuse = jp / KV_STAGES;
-          if (mbar_test_wait(&v_full[vst], vuse & 1) && mbar_test_wait(p_full, jp & 1)) {
-            tc_fence_after();
-            const uint32_t sv = smem_u32(smem + v_slot(vst));
+        if (j < nkv) {
 #pragma unroll
-            for (int k = 0; k < BKV / 16; ++k) {
-              // A = P from tensor memory (8 columns per 16 keys); B = V, which is
-              // [keys, dims] with dims contiguous: an MN-major operand whose two
-              // 64-dim panels are PANEL bytes apart (LBO), 8-key groups 1 KB apart (SBO)
-              const uint64_t bd = make_sdesc_sw128(sv + k * 16 * 128, PANEL, 1024);
-              tc_mma_f16_tmem_a(tmem + TM_O, tmem + TM_P + 8 * k, bd, idesc_pv, (jp > 0 || k > 0) ? 1u : 0u);
-            }
-            tc_commit(&v_empty[vst]);
-            tc_commit(pv_done);
-            ++jp;
-            progressed = true;
+          for (int k = 0; k < DH / 16; ++k) {
+            // A = Q_t, B = K_j, both K-major with 128-byte swizzle
+            const uint64_t off = static_cast<uint64_t>(((k >> 2) * PANEL + (k & 3) * 32) >> 4);
+            tc_mma_f16(dS, dq + off, dk0 + static_cast<uint64_t>(ks * (TILE_BYTES >> 4)) + off, idesc_qk, k > 0 ? 1u : 0u);
           }
+          tc_commit(&s_full[t]);
+          tc_commit(&k_empty[ks]);
         }
-        if (progressed) {
-          spins = 0;
-        } else if ((++spins & 255u) == 0) {
-          // bounded: give up (and let every role unwind) after the wait limit
-          const uint64_t now = globaltimer_ns();
-          if (t_idle == 0) t_idle = now;
-          if (*abort_flag) break;
-          if (now - t_idle > kWaitLimitNs) {
-            *abort_flag = 1;
-            record_error(p.err, kErrTimeout);
-            break;
-          }
-        }
-        if (progressed) t_idle = 0;
+        if (nt > 1) mbar_arrive(&turn[t ^ 1]);
       }
     }
-  } else {
-    // -------------------------------------------------- softmax warps 2..
-    const int grp = (warp - 2) >> 2;              // column group: keys / output dims [COLS grp, COLS grp + COLS)
-    const int qw = warp & 3;
+  } else if (warp >= 4) {
+    // -------------------------------------------------- softmax warps 4..11
+    const int t = (warp - 4) >> 2;                // query tile of this group
+    const int qw = warp & 3;                      // TMEM lane quarter
     const int r = qw * 32 + lane;                 // query row inside the tile == TMEM lane
-    const int col0 = grp * COLS;
     const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
+    const uint32_t tS = tmem + lane_off + TM_S + 128 * t;
+    const uint32_t tO = tmem + lane_off + TM_O + 128 * t;
     const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
     float m_ref = -INFINITY;                      // running max, log2 units
-    float l = 0.f;                                // partial row sum over this thread's columns
-    bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
-    if (ok) {
-      // stage Q row r, dims [col0, col0 + 64) (swizzle panel grp) into tensor
-      // memory: 16-byte chunk c of the row sits at (r / 8) * 1024 + (r % 8) * 128
-      // + ((c ^ (r % 8)) * 16) of the panel
-      const uint8_t* qrow = smem + OFF_Q + grp * PANEL + (r >> 3) * 1024 + (r & 7) * 128;
-      uint32_t qv[32];
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const uint4 v = *reinterpret_cast<const uint4*>(qrow + ((c ^ (r & 7)) * 16));
-        qv[4 * c + 0] = v.x; qv[4 * c + 1] = v.y; qv[4 * c + 2] = v.z; qv[4 * c + 3] = v.w;
-      }
-      tmem_st32(tmem + lane_off + TM_Q + 32 * grp, qv);
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(q_staged);
-    }
+    float l = 0.f;                                // row sum
+    bool ok = t < nt;
     for (int j = 0; ok && j < nkv; ++j) {
-      const int sb = j & 1, use = j >> 1;
-      if (!mbar_wait(&s_full[sb], use & 1, abort_flag, p.err)) { ok = false; break; }
+      if (!mbar_wait(&s_full[t], j & 1, abort_flag, p.err)) { ok = false; break; }
       tc_fence_after();
-      float s[COLS];
+      float s[BKV];
       {
-        uint32_t ra[COLS / 32][32];
+        uint32_t ra[BKV / 32][32];
 #pragma unroll
-        for (int c = 0; c < COLS / 32; ++c) tmem_ld32(tmem + lane_off + sb * 128 + col0 + 32 * c, ra[c]);
+        for (int c = 0; c < BKV / 32; ++c) tmem_ld32(tS + 32 * c, ra[c]);
         tmem_ld_wait();
 #pragma unroll
-        for (int c = 0; c < COLS / 32; ++c)
+        for (int c = 0; c < BKV / 32; ++c)
 #pragma unroll
           for (int i = 0; i < 32; ++i) s[32 * c + i] = __uint_as_float(ra[c][i]);
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s_empty[sb]);
-
-      const int valid_all = kvL - j * BKV;        // keys of this tile, >= 1
-      const int valid = valid_all - col0;         // keys of this group (may be <= 0 or >= COLS)
-      if (valid < COLS) {
+      const int valid = kvL - j * BKV;            // keys of this tile, >= 1
+      if (valid < BKV) {
 #pragma unroll
-        for (int c = 0; c < COLS; ++c) s[c] = c < valid ? s[c] : -INFINITY;
+        for (int c = 0; c < BKV; ++c) s[c] = c < valid ? s[c] : -INFINITY;
       }
-      // pairwise max tree over this group's columns, then exchange with the
-      // other groups of the row (double-buffered by tile parity, bounded wait)
-      float mx[COLS / 2];
+      // row max: eight independent chains, then a tree
+      float mx[8];
 #pragma unroll
-      for (int i = 0; i < COLS / 2; ++i) mx[i] = fmaxf(s[2 * i], s[2 * i + 1]);
+      for (int i = 0; i < 8; ++i) mx[i] = fmaxf(s[i], s[i + 8]);
 #pragma unroll
-      for (int w = COLS / 4; w >= 1; w >>= 1) {
+      for (int c = 16; c < BKV; c += 16)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mx[i] = max3(mx[i], s[c + i], s[c + 8 + i]);
+#pragma unroll
+      for (int w = 4; w >= 1; w >>= 1)
 #pragma unroll
         for (int i = 0; i < w; ++i) mx[i] = fmaxf(mx[i], mx[i + w]);
-      }
-      const float mloc = mx[0];
-      float* rm = red_max + (j & 1) * (NGRP * 128);
-      rm[grp * 128 + r] = mloc;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&max_ready[j & 1]);
-      if (!mbar_wait(&max_ready[j & 1], use & 1, abort_flag, p.err)) { ok = false; break; }
-      float mall = rm[r];
-#pragma unroll
-      for (int g = 1; g < NGRP; ++g) mall = fmaxf(mall, rm[g * 128 + r]);
-      const float mt = mall * scale_log2;
-      const float m_new = fmaxf(m_ref, mt);
+      const float m_new = fmaxf(m_ref, mx[0] * scale_log2);
       const bool need = (j == 0) || (m_new > m_ref + RESCALE_THRESHOLD);
       float alpha = 1.f;
       if (need) {
         alpha = (j == 0) ? 0.f : ex2(m_ref - m_new);
         m_ref = m_new;
       }
+      // P_t,j: keys 32c .. 32c+31 -> 16 packed columns 16c .. 16c+15 of S_t
+      // (the scores were all read above; O_t += P_t,j-1 V_j-1 has completed)
       const float neg = -m_ref;
       float rs[4] = {0.f, 0.f, 0.f, 0.f};
-      uint32_t pk[COLS / 2];
 #pragma unroll
-      for (int c = 0; c < COLS; c += 2) {
-        const float p0 = ex2(fmaf(s[c], scale_log2, neg));
-        const float p1 = ex2(fmaf(s[c + 1], scale_log2, neg));
-        rs[(c >> 1) & 3] += p0 + p1;
-        pk[c >> 1] = pack2(p0, p1, F16);
+      for (int c = 0; c < BKV / 32; ++c) {
+        uint32_t pk[16];
+        row_probs<F16>(s + 32 * c, scale_log2, neg, rs, pk);
+        tmem_st16(tS + 16 * c, pk);
       }
       l = l * alpha + ((rs[0] + rs[1]) + (rs[2] + rs[3]));
-
-      if (valid_all < BKV && grp < 2) {
-        // last, partial key tile: groups 0 and 1 clear value panels 0 and 1
-        // of the rows past kv_len so stale (possibly non-finite) data cannot
-        // meet the zero probabilities
-        const int vst = j % KV_STAGES;
-        if (!mbar_wait(&v_full[vst], (j / KV_STAGES) & 1, abort_flag, p.err)) { ok = false; break; }
-        if (r >= valid_all) {
-          uint4* v = reinterpret_cast<uint4*>(smem + v_slot(vst) + grp * PANEL + r * 128);
+      // rescale O_t in tensor memory if the reference max moved
+      if (j > 0 && __any_sync(0xffffffffu, need)) {
+#pragma unroll 1
+        for (int c = 0; c < DH / 32; ++c) {
+          uint32_t rr[32];
+          tmem_ld32(tO + 32 * c, rr);
+          tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 8; ++i) v[i] = make_uint4(0, 0, 0, 0);
+          for (int i = 0; i < 32; ++i) rr[i] = __float_as_uint(__uint_as_float(rr[i]) * alpha);
+          tmem_st32(tO + 32 * c, rr);
+        }
+      }
+      if (valid < BKV) {
+        // last, partial key tile: clear the value rows past kv_len so stale
+        // (possibly non-finite) data cannot meet the zero probabilities (both
+        // groups write the same zeros: each must see them before its PV)
+        const int vst = j % V_STAGES;
+        if (!mbar_wait(&v_full[vst], (j / V_STAGES) & 1, abort_flag, p.err)) { ok = false; break; }
+        if (r >= valid) {
+#pragma unroll
+          for (int pn = 0; pn < 2; ++pn) {
+            uint4* v = reinterpret_cast<uint4*>(smem + OFF_V + vst * TILE_BYTES + pn * PANEL + r * 128);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = make_uint4(0, 0, 0, 0);
+          }
         }
         fence_proxy_async_smem();
       }
-      if (j > 0) {
-        if (!mbar_wait(pv_done, (j - 1) & 1, abort_flag, p.err)) { ok = false; break; }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, need)) {
-#pragma unroll 1
-          for (int c = 0; c < COLS / 32; ++c) {
-            uint32_t rr[32];
-            const uint32_t ta = tmem + lane_off + 256 + col0 + 32 * c;
-            tmem_ld32(ta, rr);
-            tmem_ld_wait();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) rr[i] = __float_as_uint(__uint_as_float(rr[i]) * alpha);
-            tmem_st32(ta, rr);
-          }
-          tmem_st_wait();
-        }
-      }
-      // this thread's keys of row r -> P in tensor memory (packed pairs)
-      tmem_st32(tmem + lane_off + TM_P + 32 * grp, pk);
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(p_full);
+      if (lane == 0) mbar_arrive(&p_full[t]);
     }
-    if (ok && nkv > 0) {
-      red_sum[grp * 128 + r] = l;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(sum_ready);
-      ok = mbar_wait(sum_ready, 0, abort_flag, p.err) && mbar_wait(pv_done, (nkv - 1) & 1, abort_flag, p.err);
-    }
+    if (ok && nkv > 0) ok = mbar_wait(&o_done[t], 0, abort_flag, p.err);
     if (ok && nkv > 0) {
       tc_fence_after();
-      float lsum = 0.f;
-#pragma unroll
-      for (int g = 0; g < NGRP; ++g) lsum += red_sum[g * 128 + r];
-      const float inv_l = 1.f / lsum;
-      const int row = q0 + r;
-      const bool valid_row = (qt * BQ + r) < L;
+      const float inv_l = 1.f / l;
+      const int qrow = (qt0 + t) * BQ + r;        // row inside the segment
+      const bool valid_row = qrow < L;
       uint16_t* orow =
-          reinterpret_cast<uint16_t*>(p.out) + static_cast<size_t>(valid_row ? row : 0) * p.ldo + h * DH + col0;
+          reinterpret_cast<uint16_t*>(p.out) + static_cast<size_t>(valid_row ? seq0 + qrow : 0) * p.ldo + h * DH;
 #pragma unroll 1
-      for (int c = 0; c < COLS / 32; ++c) {
+      for (int c = 0; c < DH / 32; ++c) {
         uint32_t rr[32];
-        tmem_ld32(tmem + lane_off + 256 + col0 + 32 * c, rr);
+        tmem_ld32(tO + 32 * c, rr);
         tmem_ld_wait();
         if (valid_row) {
           uint4* dst = reinterpret_cast<uint4*>(orow + 32 * c);
@@ -403,8 +385,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
-// One block: per-segment key counts -> work units (b, h, q-tile) ordered by
-// descending kv length so the longest segments start first.
+// One block: per-segment key counts -> work units (b, h, first q-tile, tiles)
+// of up to NT query tiles, ordered by descending kv length so the longest
+// segments start first.
 __global__ void attn_schedule_kernel(const int* cu, const int* kv_len, int B, int H, int T_cap, int4* work,
                                      int* work_count, int max_units, int* err) {
   extern __shared__ int sh[];
@@ -419,7 +402,7 @@ __global__ void attn_schedule_kernel(const int* cu, const int* kv_len, int B, in
       record_error(err, kErrLayout);
       kv = 0;
     }
-    ntile[i] = (kv > 0) ? (L + BQ - 1) / BQ : 0;
+    ntile[i] = (kv > 0) ? (L + BQ * NT - 1) / (BQ * NT) : 0;   // work units (tile groups) per head
     kvs[i] = kv;
   }
   __syncthreads();
@@ -452,7 +435,11 @@ __global__ void attn_schedule_kernel(const int* cu, const int* kv_len, int B, in
     const int n = H * ntile[i];
     for (int k = threadIdx.x; k < n; k += blockDim.x) {
       const int idx = off[i] + k;
-      if (idx < max_units) work[idx] = make_int4(i, k / ntile[i], k % ntile[i], 0);
+      if (idx < max_units) {
+        const int g = k % ntile[i];
+        const int tiles = (cu[i + 1] - cu[i] + BQ - 1) / BQ;
+        work[idx] = make_int4(i, k / ntile[i], g * NT, min(NT, tiles - g * NT));
+      }
     }
   }
 }
