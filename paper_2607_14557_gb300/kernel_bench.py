@@ -1,0 +1,104 @@
+"""Microbenchmark of single hot-path kernels through the C ABI (synthetic inputs).
+
+    python -m paper_2607_14557_gb300.kernel_bench attention --lens 3100x8 [--heads 32] [--dtype f16]
+    python -m paper_2607_14557_gb300.kernel_bench linear --M 35194 --N 12288 --K 4096 [--dtype f16]
+
+Each call runs the kernel `--warmup` times, then times `--reps` calls with CUDA
+events on the launching stream and prints one JSON line (ms per call and
+TFLOP/s of the algorithmic work: 4*d*sum(L^2) for attention, 2*M*N*K for a
+linear).  Inputs are random and resident in device memory; no output is checked
+(the parity tests do that).  Used for per-kernel timings and small ncu captures.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import numpy as np
+import torch
+
+from . import seer as S
+
+
+def _lens(spec: str):
+    out = []
+    for part in spec.split(","):
+        if "x" in part:
+            length, count = part.split("x")
+            out += [int(length)] * int(count)
+        else:
+            out.append(int(part))
+    return out
+
+
+def _time(fn, warmup: int, reps: int) -> float:
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / max(reps, 1)
+
+
+def attention(args) -> dict:
+    lens = _lens(args.lens)
+    H, dh = args.heads, 128
+    D = H * dh
+    dev = torch.device("cuda", 0)
+    tdt = {"f16": torch.float16, "bf16": torch.bfloat16}[args.dtype]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    g = torch.Generator(device=dev).manual_seed(args.seed)
+    qkv = torch.randn((T, 3 * D), device=dev, dtype=torch.float32, generator=g).to(tdt)
+    o = torch.empty((T, D), device=dev, dtype=tdt)
+    cu_d = torch.as_tensor(cu).to(dev)
+    ws_bytes = S.seer_layer_workspace_size(S.make_dims(D, H, dh, 256), args.dtype, T, len(lens))
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    ms = _time(lambda: S.seer_attention(qkv, o, args.dtype, cu_d, None, len(lens), T, H, dh, ws, ws_bytes),
+               args.warmup, args.reps)
+    flops = 4.0 * D * float(np.sum(np.asarray(lens, dtype=np.float64) ** 2))
+    return {"kernel": "attention", "lens": args.lens, "heads": H, "dtype": args.dtype, "ms": ms,
+            "tflops": flops / (ms * 1e-3) / 1e12}
+
+
+def linear(args) -> dict:
+    dev = torch.device("cuda", 0)
+    tdt = {"f16": torch.float16, "bf16": torch.bfloat16}[args.dtype]
+    g = torch.Generator(device=dev).manual_seed(args.seed)
+    a = (0.5 * torch.randn((args.M, args.K), device=dev, generator=g)).to(tdt)
+    w = (0.02 * torch.randn((args.N, args.K), device=dev, generator=g)).to(tdt)
+    c = torch.empty((args.M, args.N), device=dev, dtype=tdt)
+    ms = _time(lambda: S.seer_linear(a, w, args.dtype, None, args.dtype, c, args.dtype, args.M, None, args.N, args.K),
+               args.warmup, args.reps)
+    return {"kernel": "linear", "M": args.M, "N": args.N, "K": args.K, "dtype": args.dtype, "ms": ms,
+            "tflops": 2.0 * args.M * args.N * args.K / (ms * 1e-3) / 1e12}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    sub = ap.add_subparsers(dest="kernel", required=True)
+    pa = sub.add_parser("attention")
+    pa.add_argument("--lens", default="3100x8", help="segment lengths, e.g. 3100x8 or 11900x4,500")
+    pa.add_argument("--heads", type=int, default=32)
+    pl = sub.add_parser("linear")
+    pl.add_argument("--M", type=int, default=35194)
+    pl.add_argument("--N", type=int, default=12288)
+    pl.add_argument("--K", type=int, default=4096)
+    for p in (pa, pl):
+        p.add_argument("--dtype", default="f16", choices=["f16", "bf16"])
+        p.add_argument("--warmup", type=int, default=3)
+        p.add_argument("--reps", type=int, default=10)
+        p.add_argument("--seed", type=int, default=0)
+    args = ap.parse_args(argv)
+    res = attention(args) if args.kernel == "attention" else linear(args)
+    assert S.seer_check_device() == 0, "a kernel recorded a device-side error"
+    print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()
