@@ -136,9 +136,21 @@ seer_status seer_detect_boundary(const void* x, seer_dtype dt, int T_rows, const
                                  int32_t* counts_out, int32_t* L_star_out, int32_t* i_star_out,
                                  void* stream);
 
+/* The sparsity counts alone (Sec. 3.2; S1 of seer_detect_boundary): for each
+ * response row t of each sequence, the number of |a_j| < act_eps over the F
+ * SwiGLU activations of that row with the given gate/up weights.  With
+ * accumulate != 0 the counts are added to counts_inout instead of replacing
+ * it, so several layers' gate/up weights can be tapped (a multi-layer
+ * sparsity signal, Sec. 4.5 / Table 12): the sum is then a count out of
+ * k * F for seer_snr_scan.  Arguments as for seer_detect_boundary. */
+seer_status seer_sparsity_counts(const void* x, seer_dtype dt, int T_rows, const int32_t* resp_start, int B, int N,
+                                 const void* w_gate, const void* w_up, const seer_dims* dims, float act_eps,
+                                 int accumulate, int32_t* counts_inout, void* stream);
+
 /* The SNR scan alone (Sec. 3.3) over precomputed counts: counts device int32
  * [B*N] of near-zero activations out of F; writes L_star_out (and i_star_out
- * when not NULL), device int32 [B].  Same fp64 evaluation as above. */
+ * when not NULL), device int32 [B].  Same fp64 evaluation as above.  Any
+ * look-ahead window 1 <= window <= N - 1 (params->window). */
 seer_status seer_snr_scan(const int32_t* counts, int B, int N, int F, const seer_params* params,
                           int32_t* L_star_out, int32_t* i_star_out, void* stream);
 

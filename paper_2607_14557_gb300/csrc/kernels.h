@@ -58,6 +58,9 @@ struct AttnParams {
 
 // tcgen05 / TMA kernels (16-bit operands).  Tensor maps are encoded on the host.
 int tc_gemm_smem_bytes();
+// L2 raster of the persistent GEMM (GemmParams::group_m) for a B operand of
+// b_bytes and an A row-tile of a_tile_bytes.
+int tc_gemm_group_m(long b_bytes, long a_tile_bytes);
 cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
                            const GemmParams& p, int num_sms, cudaStream_t st);
 int tc_attn_smem_bytes();

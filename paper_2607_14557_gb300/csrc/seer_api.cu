@@ -88,18 +88,6 @@ bool is16(seer_dtype dt) { return dt == SEER_BF16 || dt == SEER_F16; }
 size_t esize(seer_dtype dt) { return dt == SEER_F32 ? 4 : 2; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// L2 raster of the tcgen05 GEMM: keep the whole weight operand resident when
-// it is at most 40 MB (group_m = 1, n varies fastest), otherwise keep about
-// 24 MB of 128-row slabs of A resident while the weights stream past them.
-// Both budgets come from a sweep on GB300 at the 8B layer shapes (larger A
-// slabs thrash the L2 and re-read more, smaller ones re-stream the weights).
-int gemm_group_m(long b_bytes, long a_tile_bytes) {
-  constexpr long kResident = 40l << 20;
-  constexpr long kBudget = 24l << 20;
-  if (b_bytes <= kResident) return 1;
-  const long g = kBudget / (a_tile_bytes > 0 ? a_tile_bytes : 1);
-  return static_cast<int>(g < 1 ? 1 : (g > 4096 ? 4096 : g));
-}
 
 // ------------------------------------------------------------ TMA descriptors
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -274,7 +262,7 @@ seer_status do_linear(const void* a, const void* w, seer_dtype op_dt, const void
       return fail(SEER_ERR_UNSUPPORTED, "16-bit linear needs 16-byte aligned pointers");
     if (M_cap == 0) return SEER_OK;
     p.idesc = make_idesc(128, 256, 0, op_dt == SEER_F16);
-    p.group_m = gemm_group_m(2l * N * K, 2l * 128 * K);
+    p.group_m = tc_gemm_group_m(2l * N * K, 2l * 128 * K);
     CUtensorMap mA, mB;
     SEER_TRY(make_map16(&mA, a, op_dt, M_cap, K, K, 128));
     SEER_TRY(make_map16(&mB, w, op_dt, N, K, K, 128));
@@ -297,7 +285,8 @@ seer_status do_linear(const void* a, const void* w, seer_dtype op_dt, const void
 
 seer_status do_swiglu(const void* a, const void* wg, const void* wu, seer_dtype op_dt, void* act, seer_dtype act_dt,
                       int M_cap, const int32_t* M_dev, int F, int K, const int32_t* cu, int B, const int32_t* resp_start,
-                      int N, float act_eps, int32_t* counts, cudaStream_t st, int mode, int phase) {
+                      int N, float act_eps, int32_t* counts, cudaStream_t st, int mode, int phase,
+                      bool accumulate = false) {
   if (M_cap < 0 || F <= 0 || K <= 0) return fail(SEER_ERR_INVALID_ARG, "swiglu: bad sizes");
   if (!a || !wg || !wu) return fail(SEER_ERR_INVALID_ARG, "swiglu: null pointer");
   if (!valid_dt(op_dt) || (mode == kGemmSwiglu && !valid_dt(act_dt))) return fail(SEER_ERR_INVALID_ARG, "swiglu: unknown dtype");
@@ -331,11 +320,12 @@ seer_status do_swiglu(const void* a, const void* wg, const void* wu, seer_dtype 
   } else if (mode == kGemmSwiglu && act_dt != SEER_F32) {
     return fail(SEER_ERR_UNSUPPORTED, "fp32 swiglu needs an fp32 output");
   }
-  if (counts) SEER_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * static_cast<size_t>(B) * N, st), "memset counts");
+  if (counts && !accumulate)
+    SEER_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * static_cast<size_t>(B) * N, st), "memset counts");
   if (M_cap == 0) return SEER_OK;
   if (is16(op_dt)) {
     p.idesc = make_idesc(128, 256, 0, op_dt == SEER_F16);
-    p.group_m = gemm_group_m(2l * 2 * F * K, 2l * 128 * K);
+    p.group_m = tc_gemm_group_m(2l * 2 * F * K, 2l * 128 * K);
     CUtensorMap mA, mG, mU;
     SEER_TRY(make_map16(&mA, a, op_dt, M_cap, K, K, 128));
     SEER_TRY(make_map16(&mG, wg, op_dt, F, K, K, 128));
@@ -556,6 +546,16 @@ seer_status seer_detect_boundary(const void* x, seer_dtype dt, int T_rows, const
                             i_star_out, st),
             "snr scan launch");
   return SEER_OK;
+}
+
+seer_status seer_sparsity_counts(const void* x, seer_dtype dt, int T_rows, const int32_t* resp_start, int B, int N,
+                                 const void* w_gate, const void* w_up, const seer_dims* dims, float act_eps,
+                                 int accumulate, int32_t* counts_inout, void* stream) {
+  SEER_TRY(check_dims(dims, dt));
+  if (!x || !resp_start || !w_gate || !w_up || !counts_inout) return fail(SEER_ERR_INVALID_ARG, "counts: null pointer");
+  if (B <= 0 || N <= 0 || T_rows < N) return fail(SEER_ERR_INVALID_ARG, "counts: need B >= 1, N >= 1, T_rows >= N");
+  return do_swiglu(x, w_gate, w_up, dt, nullptr, dt, T_rows, nullptr, dims->d_ff, dims->d_model, nullptr, B, resp_start,
+                   N, act_eps, counts_inout, static_cast<cudaStream_t>(stream), kGemmCount, PH_DETECT, accumulate != 0);
 }
 
 seer_status seer_snr_scan(const int32_t* counts, int B, int N, int F, const seer_params* params, int32_t* L_star_out,

@@ -381,6 +381,19 @@ cudaError_t launch_mode(const CUtensorMap& mA, const CUtensorMap& mB0, const CUt
 
 int tc_gemm_smem_bytes() { return SMEM_BYTES; }
 
+// L2 raster of the tcgen05 GEMM: keep the whole weight operand resident when
+// it is at most 40 MB (group_m = 1, n varies fastest), otherwise keep about
+// 24 MB of 128-row slabs of A resident while the weights stream past them.
+// Both budgets come from a sweep on GB300 at the 8B layer shapes (larger A
+// slabs thrash the L2 and re-read more, smaller ones re-stream the weights).
+int tc_gemm_group_m(long b_bytes, long a_tile_bytes) {
+  constexpr long kResident = 40l << 20;
+  constexpr long kBudget = 24l << 20;
+  if (b_bytes <= kResident) return 1;
+  const long g = kBudget / (a_tile_bytes > 0 ? a_tile_bytes : 1);
+  return static_cast<int>(g < 1 ? 1 : (g > 4096 ? 4096 : g));
+}
+
 cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
                            const GemmParams& p, int num_sms, cudaStream_t st) {
   switch (mode) {

@@ -114,6 +114,17 @@ class SeerPath:
                                w.model["w_up"], self.dims, self.params, self.counts, self.L_star, self.i_star,
                                stream=stream)
 
+    def detect_multi(self, x_full, resp_start, taps: List[LayerWeights], stream=None):
+        """Boundary from a multi-layer sparsity tap (Sec. 4.5 / Table 12): the
+        near-zero counts of the response rows under each tapped layer's gate/up
+        weights are summed (a count out of len(taps) * F) and scanned once."""
+        for i, w in enumerate(taps):
+            S.seer_sparsity_counts(x_full, self.dtype, x_full.shape[0], resp_start, self.B, self.N, w.model["w_gate"],
+                                   w.model["w_up"], self.dims, self.params.act_eps, self.counts, accumulate=i > 0,
+                                   stream=stream)
+        S.seer_snr_scan(self.counts, self.B, self.N, len(taps) * self.dims.d_ff, self.params, self.L_star, self.i_star,
+                        stream=stream)
+
     def pack(self, x_full, cu_full, ctx_len, stream=None):
         self.epoch += 1
         S.seer_pack_ragged(x_full, self.dtype, cu_full, ctx_len, self.L_star, self.B, self.dims.d_model, self.N,

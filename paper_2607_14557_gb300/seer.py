@@ -69,6 +69,8 @@ def lib() -> ctypes.CDLL:
             "seer_pack_ragged": [vp, i32, vp, vp, vp, i32, i32, i32, i32, ctypes.POINTER(seer_params), vp, vp, vp,
                                  vp, vp, ctypes.c_int32, vp],
             "seer_poll_ctrl": [vp, ctypes.c_int32, i32, vp],
+            "seer_sparsity_counts": [vp, i32, i32, vp, i32, i32, vp, vp, ctypes.POINTER(seer_dims), ctypes.c_float,
+                                     i32, vp, vp],
             "seer_snr_scan": [vp, i32, i32, i32, ctypes.POINTER(seer_params), vp, vp, vp],
             "seer_layer_forward": [ctypes.POINTER(seer_layer_weights), ctypes.POINTER(seer_dims), i32, vp, vp, vp, vp,
                                    i32, i32, vp, i32, ctypes.c_float, vp, vp, sz, vp],
@@ -155,6 +157,13 @@ def seer_pack_ragged(x_full, dt, cu_full, ctx_len, L_star, B, d, N, T_capacity, 
     _check(lib().seer_pack_ragged(_p(x_full), _dt(dt), _p(cu_full), _p(ctx_len), _p(L_star), B, d, N, T_capacity,
                                   ctypes.byref(params), _p(x_packed), _p(cu_out), _p(kv_len_out), _p(meta_out),
                                   _p(host_ctrl), epoch, _stream(stream)))
+
+
+def seer_sparsity_counts(x, dt, T_rows, resp_start, B, N, w_gate, w_up, dims, act_eps, counts_inout, accumulate=False,
+                         stream=None):
+    _check(lib().seer_sparsity_counts(_p(x), _dt(dt), T_rows, _p(resp_start), B, N, _p(w_gate), _p(w_up),
+                                      ctypes.byref(dims), act_eps, 1 if accumulate else 0, _p(counts_inout),
+                                      _stream(stream)))
 
 
 def seer_snr_scan(counts, B, N, F, params, L_star_out, i_star_out=None, stream=None):

@@ -213,6 +213,49 @@ def test_snr_scan_random_matches_oracle_exactly():
     np.testing.assert_array_equal(L.cpu().numpy(), L_ref)
 
 
+@pytest.mark.parametrize("window", [1, 2, 4, 5, 7, 10])
+def test_snr_scan_window_variants_match_oracle_exactly(window):
+    # look-ahead window variants (Sec. 4.5, Table 12): plateaus of random length around the window
+    rng = _rng(40 + window)
+    B, N, F = 29, 260, 768
+    counts = rng.integers(0, 12, size=(B, N))
+    for b in range(B):
+        j = int(rng.integers(1, N - window))
+        run = int(rng.integers(1, 2 * window + 2))
+        counts[b, j:j + run] += int(rng.integers(20, 300))
+    p = S.make_params(0.0, 0.03, 0.6, window)
+    L = torch.empty(B, dtype=torch.int32, device=cuda())
+    I = torch.empty(B, dtype=torch.int32, device=cuda())
+    S.seer_snr_scan(i32(counts.ravel()), B, N, F, p, L, I)
+    i_ref, L_ref = oracle.snr_boundaries(counts, F, 0.03, 0.6, window)
+    np.testing.assert_array_equal(I.cpu().numpy(), i_ref)
+    np.testing.assert_array_equal(L.cpu().numpy(), L_ref)
+
+
+def test_multi_layer_sparsity_tap():
+    # counts of three layers' gate/up weights summed (a count out of 3F), then one scan
+    from paper_2607_14557_gb300 import driver as D
+    wl = synth.tiny_workload(dtype="bf16", seed=240, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4, window=200,
+                             boundary=("uniform", 8, 190), n_layers=3)
+    lens = synth.lengths(wl)
+    x, cu, resp = synth.hidden_full(wl, lens)
+    B, N, F = wl.batch, wl.window, wl.d_ff
+    ws = [synth.layer_weights(wl, l) for l in range(3)]
+    taps = [D.LayerWeights.from_host(w, "bf16") for w in ws]
+    path = D.SeerPath(S.make_dims(wl.d, wl.n_heads, wl.head_dim, F), "bf16", B, N, x.shape[0],
+                      S.make_params(wl.act_eps))
+    path.detect_multi(to_dev(x, "bf16"), i32(resp), taps)
+    torch.cuda.synchronize()
+    got = path.counts.cpu().numpy().reshape(B, N)
+    for b in range(B):
+        ref = sum(oracle.sparsity_counts(x[resp[b]:resp[b] + N], w["wg"], w["wu"], wl.act_eps) for w in ws)
+        assert np.abs(got[b] - ref).max() <= 0.005 * 3 * F
+    i_ref, L_ref = oracle.snr_boundaries(got, 3 * F)
+    np.testing.assert_array_equal(path.L_star.cpu().numpy(), L_ref)
+    np.testing.assert_array_equal(path.i_star.cpu().numpy(), i_ref)
+    np.testing.assert_array_equal(L_ref, lens.boundary + 1)
+
+
 # ------------------------------------------------------------------ detector end to end (S1 + S2)
 @pytest.mark.parametrize("dtype,seed", [("bf16", 1), ("bf16", 2), ("f32", 3)])
 def test_detect_boundary_planted(dtype, seed):
