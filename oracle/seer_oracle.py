@@ -36,7 +36,8 @@ __all__ = [
     "round_bf16", "round_f32", "rounding_for", "silu", "swiglu_activation", "sparsity_counts",
     "snr_boundary", "snr_boundaries", "bucket_set", "bucket_of", "padding_waste_ratio", "route",
     "segment_layout", "pack_rows", "rmsnorm", "rope", "attention_weights", "attention", "layer_forward_segment",
-    "layer_forward_packed", "layer_forward_rows", "PATH_STATIC", "PATH_VARLEN", "PATH_EAGER",
+    "layer_forward_packed", "layer_forward_rows", "kv_prefill", "layer_forward_cached", "PATH_STATIC", "PATH_VARLEN",
+    "PATH_EAGER",
 ]
 
 
@@ -341,3 +342,34 @@ def layer_forward_rows(x_seg, w, n_heads: int, rows, *, kv_len=None, dtype=None,
     if act_eps is None:
         return y
     return y, (np.abs(a_exact) < act_eps).sum(-1).astype(np.int64)
+
+
+# --------------------------------------------------------------------------
+# Prefix key/value caching combined with truncation (Sec. 4, Table 7: Seer
+# composes with KV caching of the visual + prompt prefix)
+# --------------------------------------------------------------------------
+def kv_prefill(x_prefix, w, n_heads: int, *, dtype=None, rms_eps=1e-5):
+    """Keys and values of a sequence's prefix rows for one layer (the cache):
+    the same normalisation and projections as the block, applied to the
+    prefix rows only.  Returns ``(k, v)``, each [ctx, H*dh]."""
+    R = rounding_for(dtype)
+    xn = R(rmsnorm(_f64(x_prefix), w["g_attn"], rms_eps))
+    return R(xn @ _f64(w["wk"]).T), R(xn @ _f64(w["wv"]).T)
+
+
+def layer_forward_cached(x_resp, k_prefix, v_prefix, w, n_heads: int, *, kv_valid=None, dtype=None, rms_eps=1e-5):
+    """The block over a sequence's response rows only, with the prefix keys and
+    values taken from a cache: queries are the response rows; keys/values are
+    the cached prefix rows followed by the response rows' own (the first
+    ``kv_valid`` response rows when given: bucket padding is never a key)."""
+    R = rounding_for(dtype)
+    x = _f64(x_resp)
+    nv = x.shape[0] if kv_valid is None else int(kv_valid)
+    xn = R(rmsnorm(x, w["g_attn"], rms_eps))
+    q = R(xn @ _f64(w["wq"]).T)
+    k = np.concatenate([_f64(k_prefix), R(xn[:nv] @ _f64(w["wk"]).T)])
+    v = np.concatenate([_f64(v_prefix), R(xn[:nv] @ _f64(w["wv"]).T)])
+    o = R(attention(q, k, v, n_heads))
+    h = R(x + o @ _f64(w["wo"]).T)
+    hn = R(rmsnorm(h, w["g_mlp"], rms_eps))
+    return R(h + R(swiglu_activation(hn, w["wg"], w["wu"])) @ _f64(w["wd"]).T)
