@@ -77,6 +77,17 @@ def measured_traffic(workload: int, kernel: str):
     return doc["kernels"][kernel]["traffic_bytes"]
 
 
+def graph_capacity(total: int) -> int:
+    """Smallest m * 2^e >= total with m in 8..15 (the launch capacity the pack
+    kernel reports for graph replay)."""
+    if total <= 8:
+        return 8
+    e = 0
+    while (15 << e) < total:
+        e += 1
+    return ((total + (1 << e) - 1) >> e) << e
+
+
 def layer_flops(seg, kv, d, F):
     """Algorithmic FLOPs of one layer (Eq. 2 made exact): projections 8*T*d^2,
     MLP 6*T*d*F, attention 4*d*sum(L_q * L_kv)."""
@@ -250,6 +261,31 @@ def run_stack(args, wl, world, rank, local):
         stack.step0_truncating(x_full, cu_full, resp, ctx, stream)
         ev[4].record(stream)
         torch.cuda.synchronize()
+    # prefix K/V caching composed with truncation: step 0 full, step 1 truncated
+    # with the cache prefill, steps 2..63 over the response rows only
+    resp_total = int(r["total"]) - int(lens.ctx.sum())
+    resp_cap = graph_capacity(resp_total)
+    stack.step0(x_full, cu_full, resp, ctx, stream)
+    stack.path.route()
+    stack.prefill_step(stream)
+    g_cached = stack.cached_graph(resp_cap)
+    for _ in range(max(args.warmup, 3)):
+        g_cached.replay()
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == 0
+    evc = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    with ClockSampler(local) as clk_c:
+        evc[0].record(stream)
+        stack.step0(x_full, cu_full, resp, ctx, stream)
+        evc[1].record(stream)
+        stack.path.route()
+        stack.prefill_step(stream)
+        evc[2].record(stream)
+        for _ in range(n_steps - 2):
+            g_cached.replay()
+        evc[3].record(stream)
+        torch.cuda.synchronize()
+    assert S.seer_check_device() == 0
     assert S.seer_check_device() == 0
     ms0 = ev[0].elapsed_time(ev[1])
     ms_rest = ev[1].elapsed_time(ev[2])
@@ -257,6 +293,8 @@ def run_stack(args, wl, world, rank, local):
     ms_seer = ms0 + ms_rest
     ms0_f1 = ev[3].elapsed_time(ev[4])
     dl = detect_layer + 1
+    ms_c0, ms_c1, ms_cr = evc[0].elapsed_time(evc[1]), evc[1].elapsed_time(evc[2]), evc[2].elapsed_time(evc[3])
+    ms_cached_total = ms_c0 + ms_c1 + ms_cr
     fl_full = layer_flops(lens.full, lens.full, d, F) * nl
     fl_trunc = layer_flops(seg, kv, d, F) * nl
     fl_valid = layer_flops(kv, kv, d, F) * nl
@@ -285,7 +323,16 @@ def run_stack(args, wl, world, rank, local):
             "ms_total_%d_steps" % n_steps: ms0_f1 + ms_rest, "speedup_vs_padded": ms_pad / (ms0_f1 + ms_rest),
             "ideal_ratio": fl_full * n_steps / (fl_full * dl / nl + fl_valid * (nl - dl) / nl + fl_valid * (n_steps - 1)),
             "tokens_per_s": (T_full * dl + T_valid * (nl - dl) + (n_steps - 1) * T_valid * nl) / ((ms0_f1 + ms_rest) * 1e-3)},
-        "gpu_launches": nl * 8 * (2 * n_steps) + 3 + (nl * 8 + 4), "clocks": clk.summary(),
+        "prefix_kv_cache": {
+            "ms_step0_full": ms_c0, "ms_step1_truncated_with_prefill": ms_c1,
+            "ms_steps_2_to_%d_response_rows" % (n_steps - 1): ms_cr, "ms_per_cached_step": ms_cr / (n_steps - 2),
+            "response_rows_per_step": resp_total, "launch_capacity": resp_cap,
+            "ms_total_%d_steps" % n_steps: ms_cached_total, "speedup_vs_padded": ms_pad / ms_cached_total,
+            "speedup_vs_truncated_uncached": ms_seer / ms_cached_total,
+            "tokens_per_s": (T_full + (n_steps - 1) * T_valid) * nl / (ms_cached_total * 1e-3),
+            "clocks": clk_c.summary()},
+        "gpu_launches": nl * 8 * (2 * n_steps) + 3 + (nl * 8 + 4)
+                        + (nl * 8 + 3) + nl * 13 + (n_steps - 2) * (2 + nl * 9), "clocks": clk.summary(),
         "peak_source": src,
     }
     if rank == 0:

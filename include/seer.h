@@ -282,6 +282,48 @@ seer_status seer_attention(const void* qkv, void* o, seer_dtype dt, const int32_
                            void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Prefix key/value caching combined with truncation (the paper reports that
+ * Seer composes with KV caching of the visual + prompt prefix, Table 7).
+ * A K/V cache of one layer is a [T_kv_cap, 2*H*dh] matrix (K | V per row, the
+ * layer's intermediate type: f16 for 16-bit layers, f32 for f32 ones) laid
+ * out like the packed truncated sequences: segment b owns rows
+ * [cu_kv[b], cu_kv[b+1]), its first ctx_len[b] rows hold the prefix's keys
+ * and values (seer_kv_prefill) and the rest the response rows' own, which
+ * seer_layer_forward_cached writes on every call.  cu_kv is the cu_seqlens of
+ * seer_pack_ragged.  Rotary embeddings are not supported on this path.
+ * ------------------------------------------------------------------------- */
+
+/* Fills the prefix part of a layer's K/V cache: for each segment b, the rows
+ * [cu_x[b], cu_x[b] + ctx_len[b]) of x (the layer's input hidden states, any
+ * row layout, dtype dt) are normalised and projected with the K and V rows of
+ * w->w_qkv, and the results stored at cache rows [cu_kv[b], cu_kv[b] +
+ * ctx_len[b]).  ws: seer_layer_workspace_size(dims, dt, T_x_cap, B) bytes.
+ * Row counts are read on the device; segments that would fall outside x or
+ * the cache are skipped and recorded (seer_check_device). */
+seer_status seer_kv_prefill(const seer_layer_weights* w, const seer_dims* dims, seer_dtype dt, const void* x,
+                            const int32_t* cu_x, const int32_t* ctx_len, int B, int T_x_cap, void* kv_cache,
+                            const int32_t* cu_kv, int T_kv_cap, void* ws, size_t ws_bytes, void* stream);
+
+/* The block over the response rows only (packed by cu_resp, dtype dt in and
+ * out, as from seer_gather_response): queries are the response rows, keys and
+ * values the segment's cached prefix rows followed by its response rows (the
+ * first kv_len[b] rows of the segment in all, kv_len as from
+ * seer_pack_ragged; NULL = the whole segment).  Writes the response rows'
+ * K and V into the cache first.  y_resp must not alias x_resp.  ws:
+ * seer_layer_workspace_size(dims, dt, T_resp_cap, B) bytes. */
+seer_status seer_layer_forward_cached(const seer_layer_weights* w, const seer_dims* dims, seer_dtype dt,
+                                      const void* x_resp, void* y_resp, const int32_t* cu_resp, const int32_t* ctx_len,
+                                      int B, int T_resp_cap, void* kv_cache, const int32_t* cu_kv,
+                                      const int32_t* kv_len, int T_kv_cap, void* ws, size_t ws_bytes, void* stream);
+
+/* Response rows of packed sequences: cu_resp_out[b] = cu[b] - (ctx_len[0] +
+ * ... + ctx_len[b-1]) (device int32 [B+1]) and x_resp rows [cu_resp_out[b],
+ * cu_resp_out[b+1]) = x_packed rows [cu[b] + ctx_len[b], cu[b+1]).  d * size
+ * of dt must be a multiple of 16 bytes. */
+seer_status seer_gather_response(const void* x_packed, seer_dtype dt, const int32_t* cu, const int32_t* ctx_len, int B,
+                                 int d, int T_cap, void* x_resp, int32_t* cu_resp_out, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Diagnostics.
  * ------------------------------------------------------------------------- */
 /* Thread-local message describing the last failure of this thread. */
@@ -295,10 +337,10 @@ seer_status seer_check_device(int* code_out);
 
 /* Per-phase timing with CUDA events recorded on the call's stream.
  * Phases: 0 detect GEMM, 1 SNR scan, 2 pack, 3 norm1, 4 QKV, 5 attention,
- * 6 O proj, 7 norm2, 8 gate/up, 9 down.  seer_profile_read synchronises on
- * the recorded events and returns accumulated milliseconds and launch counts
- * since the last reset. */
-#define SEER_N_PHASES 10
+ * 6 O proj, 7 norm2, 8 gate/up, 9 down, 10 K/V cache copies and prefix
+ * projections.  seer_profile_read synchronises on the recorded events and
+ * returns accumulated milliseconds and launch counts since the last reset. */
+#define SEER_N_PHASES 11
 seer_status seer_profile_enable(int on);
 seer_status seer_profile_reset(void);
 seer_status seer_profile_read(float* ms_out, int32_t* launches_out);

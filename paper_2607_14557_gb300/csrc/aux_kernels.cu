@@ -141,6 +141,66 @@ __global__ void __launch_bounds__(256) rope_kernel(void* __restrict__ qkv, const
   }
 }
 
+// ------------------------------------------------------------------ segment row copies
+// For each segment b: n rows starting at src row s0 (columns [src_c0, src_c0 +
+// row) in bytes) go to dst rows starting at d0, with
+//   s0 = src_start[b] (+ src_add[b]),  d0 = dst_start[b] (+ dst_add[b]),
+//   n  = (len ? len[b] : src_start[b+1] - src_start[b]) (- len_sub[b]).
+// A warp per row, 16-byte vectors; segments whose rows fall outside either
+// buffer are skipped and recorded.
+struct RowsCopyArgs {
+  const uint8_t* src;
+  long src_ld;                 // bytes per source row
+  int src_c0;                  // byte offset of the copied columns in a source row
+  uint8_t* dst;
+  long dst_ld;
+  int dst_c0;
+  int row;                     // bytes copied per row (multiple of 16)
+  const int* src_start;
+  const int* src_add;
+  const int* len;
+  const int* len_sub;
+  const int* dst_start;
+  const int* dst_add;
+  int B, src_rows, dst_rows;
+  int* err;
+};
+
+__global__ void __launch_bounds__(256) rows_copy_kernel(const RowsCopyArgs a) {
+  const int b = blockIdx.y;
+  const int s0 = a.src_start[b] + (a.src_add ? a.src_add[b] : 0);
+  const int d0 = a.dst_start[b] + (a.dst_add ? a.dst_add[b] : 0);
+  const int n = (a.len ? a.len[b] : a.src_start[b + 1] - a.src_start[b]) - (a.len_sub ? a.len_sub[b] : 0);
+  if (n <= 0) return;
+  if (s0 < 0 || d0 < 0 || s0 + n > a.src_rows || d0 + n > a.dst_rows) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) record_error(a.err, kErrLayout);
+    return;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int v16 = a.row / 16;
+  for (int i = blockIdx.x * 8 + warp; i < n; i += gridDim.x * 8) {
+    const uint4* sp = reinterpret_cast<const uint4*>(a.src + static_cast<size_t>(s0 + i) * a.src_ld + a.src_c0);
+    uint4* dp = reinterpret_cast<uint4*>(a.dst + static_cast<size_t>(d0 + i) * a.dst_ld + a.dst_c0);
+    for (int v = lane; v < v16; v += 32) dp[v] = sp[v];
+  }
+}
+
+// cu_ctx = exclusive prefix sums of ctx (B+1 entries); cu_resp[b] = cu[b] -
+// cu_ctx[b]: the offsets of the rows past each segment's first ctx[b] rows.
+__global__ void resp_layout_kernel(const int* cu, const int* ctx, int B, int* cu_resp, int* cu_ctx, int* err) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  int acc = 0;
+  for (int b = 0; b <= B; ++b) {
+    if (cu_ctx) cu_ctx[b] = acc;
+    if (cu_resp && cu) {
+      const int r = cu[b] - acc;
+      if (r < 0 || (b > 0 && ctx[b - 1] > cu[b] - cu[b - 1])) record_error(err, kErrLayout);
+      cu_resp[b] = r < 0 ? 0 : r;
+    }
+    if (b < B) acc += ctx[b];
+  }
+}
+
 // ------------------------------------------------------------------ SNR scan
 // Sec. 3.3: first 0-based i in [1, N-w] with
 //   jump  = min(s_i .. s_{i+w-1}) - s_{i-1} >= tau_jump
@@ -387,6 +447,27 @@ cudaError_t launch_rope(void* qkv, int type, const int* cu, int B, int T_cap, in
     case kBF16: rope_kernel<kBF16><<<blocks, 256, 0, st>>>(qkv, cu, B, T_cap, n_heads, head_dim, theta, err); break;
     default: return cudaErrorInvalidValue;
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rows_copy(const void* src, long src_ld, int src_c0, void* dst, long dst_ld, int dst_c0, int row_bytes,
+                             const int* src_start, const int* src_add, const int* len, const int* len_sub,
+                             const int* dst_start, const int* dst_add, int B, int src_rows, int dst_rows, int max_rows,
+                             int* err, cudaStream_t st) {
+  if (B <= 0 || row_bytes <= 0 || max_rows <= 0) return cudaSuccess;
+  if (row_bytes % 16 != 0 || src_c0 % 16 != 0 || dst_c0 % 16 != 0 || src_ld % 16 != 0 || dst_ld % 16 != 0 ||
+      (reinterpret_cast<uintptr_t>(src) & 15u) != 0 || (reinterpret_cast<uintptr_t>(dst) & 15u) != 0)
+    return cudaErrorInvalidValue;
+  RowsCopyArgs a{static_cast<const uint8_t*>(src), src_ld, src_c0, static_cast<uint8_t*>(dst), dst_ld, dst_c0, row_bytes,
+                 src_start, src_add, len, len_sub, dst_start, dst_add, B, src_rows, dst_rows, err};
+  const int gx = (max_rows + 7) / 8 < 64 ? (max_rows + 7) / 8 : 64;
+  rows_copy_kernel<<<dim3(gx, B), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_resp_layout(const int* cu, const int* ctx, int B, int* cu_resp, int* cu_ctx, int* err,
+                               cudaStream_t st) {
+  resp_layout_kernel<<<1, 32, 0, st>>>(cu, ctx, B, cu_resp, cu_ctx, err);
   return cudaGetLastError();
 }
 

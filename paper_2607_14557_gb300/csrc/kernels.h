@@ -43,8 +43,12 @@ struct GemmParams {
 };
 
 struct AttnParams {
-  const int* cu;          // [B+1]
-  const int* kv_len;      // [B] or null
+  const int* cu;          // [B+1] query segment offsets (rows of the q source)
+  const int* kv_len;      // [B] keys per segment, or null (= the K/V segment length)
+  const int* cu_kv;       // [B+1] K/V segment offsets, or null (= cu: q, k, v share rows)
+  const void* kv;         // K/V rows (fp32 path), or null (= the qkv buffer)
+  int ld_kv;              // elements per K/V row
+  int xk0, xv0;           // column of head 0's K and V inside a K/V row
   int B;
   int T_cap;
   int n_heads;
@@ -64,9 +68,10 @@ int tc_gemm_group_m(long b_bytes, long a_tile_bytes);
 cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
                            const GemmParams& p, int num_sms, cudaStream_t st);
 int tc_attn_smem_bytes();
-cudaError_t launch_tc_attn(const CUtensorMap& mQKV, const AttnParams& p, int grid, bool f16, cudaStream_t st);
-cudaError_t launch_attn_schedule(const int* cu, const int* kv_len, int B, int n_heads, int T_cap, int4* work,
-                                 int* work_count, int max_units, int* err, cudaStream_t st);
+cudaError_t launch_tc_attn(const CUtensorMap& mQ, const CUtensorMap& mKV, const AttnParams& p, int grid, bool f16,
+                           cudaStream_t st);
+cudaError_t launch_attn_schedule(const int* cu, const int* cu_kv, const int* kv_len, int B, int n_heads, int T_cap,
+                                 int4* work, int* work_count, int max_units, int* err, cudaStream_t st);
 
 // CUDA-core kernels (fp32 storage; small shapes).
 cudaError_t launch_simt_gemm(int mode, const float* A, const float* B0, const float* B1, const GemmParams& p,
@@ -78,6 +83,17 @@ cudaError_t launch_rmsnorm(const void* x, int in_type, const void* g, void* y, i
                            const int* M_dev, int d, float eps, int* err, cudaStream_t st);
 cudaError_t launch_rope(void* qkv, int type, const int* cu, int B, int T_cap, int n_heads, int head_dim, float theta,
                         int* err, int num_sms, cudaStream_t st);
+// Per-segment row copies (see aux_kernels.cu): rows of segment b go from src
+// rows src_start[b] (+ src_add[b]) to dst rows dst_start[b] (+ dst_add[b]);
+// n = (len ? len[b] : src_start[b+1] - src_start[b]) (- len_sub[b]).
+// Offsets and sizes in bytes; max_rows bounds any segment's n (grid size).
+cudaError_t launch_rows_copy(const void* src, long src_ld, int src_c0, void* dst, long dst_ld, int dst_c0, int row_bytes,
+                             const int* src_start, const int* src_add, const int* len, const int* len_sub,
+                             const int* dst_start, const int* dst_add, int B, int src_rows, int dst_rows, int max_rows,
+                             int* err, cudaStream_t st);
+// cu_ctx = exclusive sums of ctx; cu_resp[b] = cu[b] - cu_ctx[b] (either output may be null).
+cudaError_t launch_resp_layout(const int* cu, const int* ctx, int B, int* cu_resp, int* cu_ctx, int* err,
+                               cudaStream_t st);
 cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, cudaStream_t st);
 cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,
                             int* L_star, int* i_star, cudaStream_t st);

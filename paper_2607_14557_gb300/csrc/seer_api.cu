@@ -160,7 +160,7 @@ class Phase {
   cudaEvent_t a_ = nullptr, b_ = nullptr;
 };
 
-enum { PH_DETECT = 0, PH_SCAN, PH_PACK, PH_NORM1, PH_QKV, PH_ATTN, PH_OPROJ, PH_NORM2, PH_GATEUP, PH_DOWN };
+enum { PH_DETECT = 0, PH_SCAN, PH_PACK, PH_NORM1, PH_QKV, PH_ATTN, PH_OPROJ, PH_NORM2, PH_GATEUP, PH_DOWN, PH_KV };
 
 // ------------------------------------------------------------ workspace
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -358,9 +358,22 @@ seer_status do_rmsnorm(const void* x, seer_dtype x_dt, const void* g, void* y, s
   return SEER_OK;
 }
 
+// Where an attention call finds its keys and values (default: the K and V
+// column blocks of the qkv buffer itself, rows shared with the queries).
+struct KvSource {
+  const void* kv = nullptr;      // [T_kv_cap, ld] rows holding K | V
+  int ld = 0;                    // elements per row
+  int xk0 = 0, xv0 = 0;          // columns of head 0's K and V
+  const int32_t* cu_kv = nullptr;
+  int T_kv_cap = 0;
+};
+
 seer_status do_attention(const void* qkv, void* o, seer_dtype dt, const int32_t* cu, const int32_t* kv_len, int B,
-                         int T_cap, int H, int dh, void* sched, size_t sched_bytes, cudaStream_t st) {
+                         int T_cap, int H, int dh, void* sched, size_t sched_bytes, cudaStream_t st,
+                         const KvSource& kvs = KvSource()) {
   if (!qkv || !o || !cu) return fail(SEER_ERR_INVALID_ARG, "attention: null pointer");
+  if (kvs.kv && (!kvs.cu_kv || kvs.T_kv_cap < 0 || kvs.ld < 2 * H * dh))
+    return fail(SEER_ERR_INVALID_ARG, "attention: a separate K/V source needs cu_kv, a capacity and rows of >= 2*H*dh");
   if (B <= 0 || T_cap < 0 || H <= 0 || dh <= 0) return fail(SEER_ERR_INVALID_ARG, "attention: bad sizes");
   if (!valid_dt(dt)) return fail(SEER_ERR_INVALID_ARG, "attention: unknown dtype");
   DeviceInfo* di;
@@ -375,8 +388,15 @@ seer_status do_attention(const void* qkv, void* o, seer_dtype dt, const int32_t*
   p.out = o;
   p.ldo = H * dh;
   p.err = di->err;
+  p.kv = kvs.kv;
+  p.cu_kv = kvs.kv ? kvs.cu_kv : nullptr;
+  p.ld_kv = kvs.kv ? kvs.ld : 3 * H * dh;
+  p.xk0 = kvs.kv ? kvs.xk0 : H * dh;
+  p.xv0 = kvs.kv ? kvs.xv0 : 2 * H * dh;
   if (is16(dt)) {
     if (dh != 128) return fail(SEER_ERR_UNSUPPORTED, "16-bit attention needs head_dim == 128");
+    if (kvs.kv && (!aligned16(kvs.kv) || (static_cast<long>(kvs.ld) * 2) % 16 != 0 || kvs.xk0 % 64 != 0 || kvs.xv0 % 64 != 0))
+      return fail(SEER_ERR_UNSUPPORTED, "attention: K/V rows must be 16-byte aligned with 64-element column offsets");
     const size_t need = attn_sched_bytes(T_cap, B, H);
     if (!sched || sched_bytes < need)
       return fail(SEER_ERR_WORKSPACE, "attention needs %zu bytes of schedule workspace", need);
@@ -388,11 +408,13 @@ seer_status do_attention(const void* qkv, void* o, seer_dtype dt, const int32_t*
     int* count = reinterpret_cast<int*>(static_cast<uint8_t*>(sched) + align256(static_cast<size_t>(max_units) * sizeof(int4)));
     p.work = work;
     p.work_count = count;
-    CUtensorMap m;
+    CUtensorMap m, mkv;
     SEER_TRY(make_map16(&m, qkv, dt, T_cap, 3 * H * dh, 3 * H * dh, 128));
+    if (kvs.kv) SEER_TRY(make_map16(&mkv, kvs.kv, dt, kvs.T_kv_cap > 0 ? kvs.T_kv_cap : 1, kvs.ld, kvs.ld, 128));
     Phase ph(PH_ATTN, st);
-    SEER_CUDA(launch_attn_schedule(cu, kv_len, B, H, T_cap, work, count, max_units, di->err, st), "attn schedule");
-    SEER_CUDA(launch_tc_attn(m, p, max_units, dt == SEER_F16, st), "tc_attn launch");
+    SEER_CUDA(launch_attn_schedule(cu, p.cu_kv, kv_len, B, H, T_cap, work, count, max_units, di->err, st),
+              "attn schedule");
+    SEER_CUDA(launch_tc_attn(m, kvs.kv ? mkv : m, p, max_units, dt == SEER_F16, st), "tc_attn launch");
   } else {
     if (dh > 128 || dh % 4 != 0) return fail(SEER_ERR_UNSUPPORTED, "fp32 attention needs head_dim <= 128, %% 4 == 0");
     if (T_cap == 0) return SEER_OK;
@@ -667,6 +689,125 @@ seer_status seer_layer_forward(const seer_layer_weights* w, const seer_dims* dim
   SEER_TRY(do_swiglu(xn, w->w_gate, w->w_up, it, act, it, T_capacity, M_dev, F, d, cu_seqlens, B, count_resp_start, N,
                      act_eps, count_resp_start ? counts_out : nullptr, st, kGemmSwiglu, PH_GATEUP));
   SEER_TRY(do_linear(act, w->w_down, it, h, it, y, dt, T_capacity, M_dev, d, F, st, PH_DOWN));
+  return SEER_OK;
+}
+
+
+seer_status seer_gather_response(const void* x_packed, seer_dtype dt, const int32_t* cu, const int32_t* ctx_len, int B,
+                                 int d, int T_cap, void* x_resp, int32_t* cu_resp_out, void* stream) {
+  if (!valid_dt(dt)) return fail(SEER_ERR_INVALID_ARG, "gather: unknown dtype");
+  if (!x_packed || !cu || !ctx_len || !x_resp || !cu_resp_out) return fail(SEER_ERR_INVALID_ARG, "gather: null pointer");
+  if (B <= 0 || d <= 0 || T_cap < 0) return fail(SEER_ERR_INVALID_ARG, "gather: bad sizes");
+  const long row = static_cast<long>(d) * static_cast<long>(esize(dt));
+  if (row % 16 != 0 || !aligned16(x_packed) || !aligned16(x_resp))
+    return fail(SEER_ERR_UNSUPPORTED, "gather: 16-byte aligned rows required");
+  DeviceInfo* di;
+  SEER_TRY(device_info(&di));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Phase ph(PH_KV, st);
+  SEER_CUDA(launch_resp_layout(cu, ctx_len, B, cu_resp_out, nullptr, di->err, st), "response layout");
+  SEER_CUDA(launch_rows_copy(x_packed, row, 0, x_resp, row, 0, static_cast<int>(row), cu, ctx_len, nullptr, ctx_len,
+                             cu_resp_out, nullptr, B, T_cap, T_cap, T_cap, di->err, st),
+            "response gather");
+  return SEER_OK;
+}
+
+seer_status seer_kv_prefill(const seer_layer_weights* w, const seer_dims* dims, seer_dtype dt, const void* x,
+                            const int32_t* cu_x, const int32_t* ctx_len, int B, int T_x_cap, void* kv_cache,
+                            const int32_t* cu_kv, int T_kv_cap, void* ws, size_t ws_bytes, void* stream) {
+  SEER_TRY(check_dims(dims, dt));
+  if (!w || !w->w_qkv || !w->g_attn) return fail(SEER_ERR_INVALID_ARG, "prefill: null weight pointer");
+  if (!x || !cu_x || !ctx_len || !kv_cache || !cu_kv) return fail(SEER_ERR_INVALID_ARG, "prefill: null pointer");
+  if (B <= 0 || T_x_cap < 0 || T_kv_cap < 0) return fail(SEER_ERR_INVALID_ARG, "prefill: bad sizes");
+  if (dims->rope_theta != 0.f) return fail(SEER_ERR_UNSUPPORTED, "the K/V cache path has no rotary embedding");
+  const LayerWs L = layer_ws(*dims, dt, T_x_cap, B);
+  if (!ws || ws_bytes < L.total) return fail(SEER_ERR_WORKSPACE, "prefill needs %zu bytes of workspace", L.total);
+  if (!aligned16(ws) || !aligned16(x) || !aligned16(kv_cache)) return fail(SEER_ERR_UNSUPPORTED, "prefill needs 16-byte aligned pointers");
+  if (T_x_cap == 0) return SEER_OK;
+  DeviceInfo* di;
+  SEER_TRY(device_info(&di));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int d = dims->d_model, D2 = 2 * dims->n_heads * dims->head_dim;
+  const seer_dtype it = dt == SEER_F32 ? SEER_F32 : SEER_F16;
+  const long xrow = static_cast<long>(d) * esize(dt), irow = static_cast<long>(d) * esize(it);
+  const long kvrow = static_cast<long>(D2) * esize(it);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  void* xp = base + L.off_h;                     // prefix rows, packed  [sum ctx, d]
+  void* xn = base + L.off_xn;                    // normalised           [sum ctx, d]
+  void* kvp = base + L.off_qkv;                  // their K | V          [sum ctx, 2D]
+  int32_t* cu_ctx = reinterpret_cast<int32_t*>(base + L.off_sched);   // [B+1], before the (unused) schedule
+  {
+    Phase ph(PH_KV, st);
+    SEER_CUDA(launch_resp_layout(nullptr, ctx_len, B, nullptr, cu_ctx, di->err, st), "prefix layout");
+    SEER_CUDA(launch_rows_copy(x, xrow, 0, xp, xrow, 0, static_cast<int>(xrow), cu_x, nullptr, ctx_len, nullptr, cu_ctx,
+                               nullptr, B, T_x_cap, T_x_cap, T_x_cap, di->err, st),
+              "prefix gather");
+  }
+  SEER_TRY(do_rmsnorm(xp, dt, w->g_attn, xn, it, T_x_cap, cu_ctx + B, d, dims->rms_eps, st, PH_KV));
+  const void* w_kv = static_cast<const uint8_t*>(w->w_qkv) + static_cast<size_t>(D2 / 2) * d * esize(it);
+  SEER_TRY(do_linear(xn, w_kv, it, nullptr, it, kvp, it, T_x_cap, cu_ctx + B, D2, d, st, PH_KV));
+  Phase ph(PH_KV, st);
+  SEER_CUDA(launch_rows_copy(kvp, kvrow, 0, kv_cache, kvrow, 0, static_cast<int>(kvrow), cu_ctx, nullptr, nullptr, nullptr,
+                             cu_kv, nullptr, B, T_x_cap, T_kv_cap, T_x_cap, di->err, st),
+            "prefix K/V scatter");
+  return SEER_OK;
+}
+
+seer_status seer_layer_forward_cached(const seer_layer_weights* w, const seer_dims* dims, seer_dtype dt,
+                                      const void* x_resp, void* y_resp, const int32_t* cu_resp, const int32_t* ctx_len,
+                                      int B, int T_resp_cap, void* kv_cache, const int32_t* cu_kv,
+                                      const int32_t* kv_len, int T_kv_cap, void* ws, size_t ws_bytes, void* stream) {
+  SEER_TRY(check_dims(dims, dt));
+  if (!w || !w->w_qkv || !w->w_o || !w->w_gate || !w->w_up || !w->w_down || !w->g_attn || !w->g_mlp)
+    return fail(SEER_ERR_INVALID_ARG, "cached layer: null weight pointer");
+  if (!x_resp || !y_resp || !cu_resp || !ctx_len || !kv_cache || !cu_kv)
+    return fail(SEER_ERR_INVALID_ARG, "cached layer: null pointer");
+  if (x_resp == y_resp) return fail(SEER_ERR_INVALID_ARG, "cached layer: y must not alias x");
+  if (B <= 0 || T_resp_cap < 0 || T_kv_cap < 0) return fail(SEER_ERR_INVALID_ARG, "cached layer: bad sizes");
+  if (dims->rope_theta != 0.f) return fail(SEER_ERR_UNSUPPORTED, "the K/V cache path has no rotary embedding");
+  const LayerWs L = layer_ws(*dims, dt, T_resp_cap, B);
+  if (!ws || ws_bytes < L.total) return fail(SEER_ERR_WORKSPACE, "cached layer needs %zu bytes of workspace", L.total);
+  if (!aligned16(ws) || !aligned16(x_resp) || !aligned16(y_resp) || !aligned16(kv_cache))
+    return fail(SEER_ERR_UNSUPPORTED, "cached layer needs 16-byte aligned pointers");
+  if (T_resp_cap == 0) return SEER_OK;
+  DeviceInfo* di;
+  SEER_TRY(device_info(&di));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int d = dims->d_model, F = dims->d_ff, H = dims->n_heads, dh = dims->head_dim, D = H * dh;
+  const seer_dtype it = dt == SEER_F32 ? SEER_F32 : SEER_F16;
+  const long es = static_cast<long>(esize(it));
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  void* xn = base + L.off_xn;
+  void* qkv = base + L.off_qkv;
+  void* h = base + L.off_h;
+  void* act = base + L.off_act;
+  void* sched = base + L.off_sched;
+  const int32_t* M_dev = cu_resp + B;
+  const float eps = dims->rms_eps;
+
+  SEER_TRY(do_rmsnorm(x_resp, dt, w->g_attn, xn, it, T_resp_cap, M_dev, d, eps, st, PH_NORM1));
+  SEER_TRY(do_linear(xn, w->w_qkv, it, nullptr, it, qkv, it, T_resp_cap, M_dev, 3 * d, d, st, PH_QKV));
+  {
+    // the response rows' K | V into the cache, after each segment's prefix
+    Phase ph(PH_KV, st);
+    SEER_CUDA(launch_rows_copy(qkv, 3 * D * es, static_cast<int>(D * es), kv_cache, 2 * D * es, 0,
+                               static_cast<int>(2 * D * es), cu_resp, nullptr, nullptr, nullptr, cu_kv, ctx_len, B,
+                               T_resp_cap, T_kv_cap, T_resp_cap, di->err, st),
+              "response K/V scatter");
+  }
+  KvSource kvs;
+  kvs.kv = kv_cache;
+  kvs.ld = 2 * D;
+  kvs.xk0 = 0;
+  kvs.xv0 = D;
+  kvs.cu_kv = cu_kv;
+  kvs.T_kv_cap = T_kv_cap;
+  SEER_TRY(do_attention(qkv, xn, it, cu_resp, kv_len, B, T_resp_cap, H, dh, sched, L.total - L.off_sched, st, kvs));
+  SEER_TRY(do_linear(xn, w->w_o, it, x_resp, dt, h, it, T_resp_cap, M_dev, d, d, st, PH_OPROJ));
+  SEER_TRY(do_rmsnorm(h, it, w->g_mlp, xn, it, T_resp_cap, M_dev, d, eps, st, PH_NORM2));
+  SEER_TRY(do_swiglu(xn, w->w_gate, w->w_up, it, act, it, T_resp_cap, M_dev, F, d, cu_resp, B, nullptr, 0, 0.f, nullptr,
+                     st, kGemmSwiglu, PH_GATEUP));
+  SEER_TRY(do_linear(act, w->w_down, it, h, it, y_resp, dt, T_resp_cap, M_dev, d, F, st, PH_DOWN));
   return SEER_OK;
 }
 

@@ -149,12 +149,14 @@ __global__ void __launch_bounds__(256) simt_attn_kernel(const float* __restrict_
     if (p.cu[mid] <= row) lo = mid; else hi = mid;
   }
   const int seq0 = p.cu[lo];
-  const int L = p.cu[lo + 1] - seq0;
-  const int kvL = p.kv_len ? p.kv_len[lo] : L;
-  if (kvL <= 0 || kvL > L) {
+  const int kv0 = p.cu_kv ? p.cu_kv[lo] : seq0;
+  const int Lkv = p.cu_kv ? p.cu_kv[lo + 1] - kv0 : p.cu[lo + 1] - seq0;
+  const int kvL = p.kv_len ? p.kv_len[lo] : Lkv;
+  if (kvL <= 0 || kvL > Lkv) {
     if (lane == 0) record_error(p.err, kErrLayout);
     return;
   }
+  const float* kvsrc = p.kv ? static_cast<const float*>(p.kv) : qkv;
   const int per = (dh + 31) / 32;   // <= 4
   float q[4], o[4];
   const float* qrow = qkv + static_cast<size_t>(row) * 3 * D + h * dh;
@@ -166,8 +168,9 @@ __global__ void __launch_bounds__(256) simt_attn_kernel(const float* __restrict_
   const float scale = 1.0f / sqrtf(static_cast<float>(dh));
   float m = -INFINITY, l = 0.f;
   for (int kidx = 0; kidx < kvL; ++kidx) {
-    const float* krow = qkv + static_cast<size_t>(seq0 + kidx) * 3 * D + D + h * dh;
-    const float* vrow = krow + D;
+    const float* kvrow = kvsrc + static_cast<size_t>(kv0 + kidx) * p.ld_kv;
+    const float* krow = kvrow + p.xk0 + h * dh;
+    const float* vrow = kvrow + p.xv0 + h * dh;
     float part = 0.f;
     for (int i = 0; i < per; ++i) {
       const int c = lane + 32 * i;

@@ -113,7 +113,7 @@ __device__ __forceinline__ void row_probs(const float* s, float scale_log2, floa
 
 template <bool F16>
 __global__ void __launch_bounds__(THREADS, 1)
-    tc_attn_kernel(const __grid_constant__ CUtensorMap mQKV, const AttnParams p) {
+    tc_attn_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mKV, const AttnParams p) {
   const int u = blockIdx.x;
   if (u >= *p.work_count) return;
   const int4 wk = p.work[u];
@@ -122,9 +122,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int L = p.cu[b + 1] - seq0;
   const int kvL = p.kv_len ? p.kv_len[b] : L;
   const int q0 = seq0 + qt0 * BQ;
+  const int kv0 = p.cu_kv ? p.cu_kv[b] : seq0;  // first K/V row of the segment
   const int nkv = (kvL + BKV - 1) / BKV;
-  const int D = p.n_heads * DH;
-  const int xq = h * DH, xk = D + h * DH, xv = 2 * D + h * DH;
+  const int xq = h * DH, xk = p.xk0 + h * DH, xv = p.xv0 + h * DH;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -174,11 +174,12 @@ __global__ void __launch_bounds__(THREADS, 1)
     // lane 0 loads Q and the K tiles, lane 1 the V tiles, so waiting for a V
     // buffer (freed by PV) never delays the next K (needed by QK^T).
     if (lane == 0) {
-      tma_prefetch_desc(&mQKV);
+      tma_prefetch_desc(&mQ);
+      tma_prefetch_desc(&mKV);
       mbar_arrive_expect_tx(q_full, nt * TILE_BYTES);
       for (int t = 0; t < nt; ++t) {
-        tma_load_2d(smem + OFF_Q + t * TILE_BYTES, &mQKV, q_full, xq, q0 + t * BQ);
-        tma_load_2d(smem + OFF_Q + t * TILE_BYTES + PANEL, &mQKV, q_full, xq + 64, q0 + t * BQ);
+        tma_load_2d(smem + OFF_Q + t * TILE_BYTES, &mQ, q_full, xq, q0 + t * BQ);
+        tma_load_2d(smem + OFF_Q + t * TILE_BYTES + PANEL, &mQ, q_full, xq + 64, q0 + t * BQ);
       }
     }
     if (lane < 2) {
@@ -193,8 +194,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (use > 0 && !mbar_wait(&empty[st], (use - 1) & 1, abort_flag, p.err)) break;
         uint8_t* dst = smem + (is_k ? OFF_K : OFF_V) + st * TILE_BYTES;
         mbar_arrive_expect_tx(&full[st], TILE_BYTES);
-        tma_load_2d(dst, &mQKV, &full[st], x, seq0 + j * BKV);
-        tma_load_2d(dst + PANEL, &mQKV, &full[st], x + 64, seq0 + j * BKV);
+        tma_load_2d(dst, &mKV, &full[st], x, kv0 + j * BKV);
+        tma_load_2d(dst + PANEL, &mKV, &full[st], x + 64, kv0 + j * BKV);
         ++issued;
       }
       if (*abort_flag) {
@@ -388,8 +389,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 // One block: per-segment key counts -> work units (b, h, first q-tile, tiles)
 // of up to NT query tiles, ordered by descending kv length so the longest
 // segments start first.
-__global__ void attn_schedule_kernel(const int* cu, const int* kv_len, int B, int H, int T_cap, int4* work,
-                                     int* work_count, int max_units, int* err) {
+__global__ void attn_schedule_kernel(const int* cu, const int* cu_kv, const int* kv_len, int B, int H, int T_cap,
+                                     int4* work, int* work_count, int max_units, int* err) {
   extern __shared__ int sh[];
   int* ntile = sh;           // [B]
   int* kvs = sh + B;         // [B]
@@ -397,8 +398,9 @@ __global__ void attn_schedule_kernel(const int* cu, const int* kv_len, int B, in
   int* rank = sh + 3 * B;    // [B]
   for (int i = threadIdx.x; i < B; i += blockDim.x) {
     const int L = cu[i + 1] - cu[i];
-    int kv = kv_len ? kv_len[i] : L;
-    if (L < 0 || cu[i] < 0 || cu[i + 1] > T_cap || kv > L || (L > 0 && kv <= 0)) {
+    const int Lkv = cu_kv ? cu_kv[i + 1] - cu_kv[i] : L;   // rows of the segment's K/V
+    int kv = kv_len ? kv_len[i] : Lkv;
+    if (L < 0 || cu[i] < 0 || cu[i + 1] > T_cap || kv > Lkv || (L > 0 && kv <= 0)) {
       record_error(err, kErrLayout);
       kv = 0;
     }
@@ -445,7 +447,7 @@ __global__ void attn_schedule_kernel(const int* cu, const int* kv_len, int B, in
 }
 
 template <bool F16>
-cudaError_t launch_typed(const CUtensorMap& mQKV, const AttnParams& p, int grid, cudaStream_t st) {
+cudaError_t launch_typed(const CUtensorMap& mQ, const CUtensorMap& mKV, const AttnParams& p, int grid, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(tc_attn_kernel<F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
@@ -453,7 +455,7 @@ cudaError_t launch_typed(const CUtensorMap& mQKV, const AttnParams& p, int grid,
     attr_set = true;
   }
   if (grid <= 0) return cudaSuccess;
-  tc_attn_kernel<F16><<<grid, THREADS, SMEM_BYTES, st>>>(mQKV, p);
+  tc_attn_kernel<F16><<<grid, THREADS, SMEM_BYTES, st>>>(mQ, mKV, p);
   return cudaGetLastError();
 }
 
@@ -461,19 +463,20 @@ cudaError_t launch_typed(const CUtensorMap& mQKV, const AttnParams& p, int grid,
 
 int tc_attn_smem_bytes() { return SMEM_BYTES; }
 
-cudaError_t launch_tc_attn(const CUtensorMap& mQKV, const AttnParams& p, int grid, bool f16, cudaStream_t st) {
-  return f16 ? launch_typed<true>(mQKV, p, grid, st) : launch_typed<false>(mQKV, p, grid, st);
+cudaError_t launch_tc_attn(const CUtensorMap& mQ, const CUtensorMap& mKV, const AttnParams& p, int grid, bool f16,
+                           cudaStream_t st) {
+  return f16 ? launch_typed<true>(mQ, mKV, p, grid, st) : launch_typed<false>(mQ, mKV, p, grid, st);
 }
 
-cudaError_t launch_attn_schedule(const int* cu, const int* kv_len, int B, int n_heads, int T_cap, int4* work,
-                                 int* work_count, int max_units, int* err, cudaStream_t st) {
+cudaError_t launch_attn_schedule(const int* cu, const int* cu_kv, const int* kv_len, int B, int n_heads, int T_cap,
+                                 int4* work, int* work_count, int max_units, int* err, cudaStream_t st) {
   const size_t sm = static_cast<size_t>(4) * B * sizeof(int);
   if (sm > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(attn_schedule_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(sm));
     if (e != cudaSuccess) return e;
   }
-  attn_schedule_kernel<<<1, 256, sm, st>>>(cu, kv_len, B, n_heads, T_cap, work, work_count, max_units, err);
+  attn_schedule_kernel<<<1, 256, sm, st>>>(cu, cu_kv, kv_len, B, n_heads, T_cap, work, work_count, max_units, err);
   return cudaGetLastError();
 }
 

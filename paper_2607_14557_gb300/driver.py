@@ -214,6 +214,8 @@ class SeerStack:
         self.hook_counts = torch.zeros(B * N, dtype=torch.int32, device=dev)
         self.graphs: Dict[object, torch.cuda.CUDAGraph] = {}
         self.h_packed: Optional[torch.Tensor] = None
+        self.kv_cache: Optional[List[torch.Tensor]] = None
+        self.ctx_len: Optional[torch.Tensor] = None
 
     def _run_layers(self, x, cu, kv, T_cap, resp_start=None, stream=None, n_layers=None, start=0):
         p = self.path
@@ -233,6 +235,7 @@ class SeerStack:
     def step0(self, x_full, cu_full, resp_start, ctx_len, stream=None):
         """Full-window step with the fused count hook, then detect + route/pack."""
         p = self.path
+        self.ctx_len = ctx_len
         out = self._run_layers(x_full, cu_full, None, p.T_full, resp_start=resp_start, stream=stream)
         p.detect(x_full, resp_start, self.layers[self.detect_layer], stream)
         p.pack(x_full, cu_full, ctx_len, stream)
@@ -247,6 +250,7 @@ class SeerStack:
         packed too (input of the later steps).  Returns the last layer's output
         in the packed layout."""
         p = self.path
+        self.ctx_len = ctx_len
         h = self._run_layers(x_full, cu_full, None, p.T_full, resp_start=resp_start, stream=stream,
                              n_layers=self.detect_layer + 1)
         p.detect(x_full, resp_start, self.layers[self.detect_layer], stream)
@@ -279,6 +283,60 @@ class SeerStack:
             fn(stream=torch.cuda.current_stream())
         self.graphs[key] = g
         return g
+
+    # ------------------------------------------------------------ prefix K/V cache
+    def _cache_buffers(self):
+        """Per-layer K/V caches [T_full, 2*H*dh] in the layers' intermediate
+        type (packed truncated layout) and the response-row buffers."""
+        p = self.path
+        if self.kv_cache is None:
+            dev = p.device
+            it = torch.float32 if p.dtype == "f32" else torch.float16
+            D = p.dims.n_heads * p.dims.head_dim
+            self.kv_cache = [torch.empty((p.T_full, 2 * D), dtype=it, device=dev) for _ in self.layers]
+            self.resp = [torch.empty_like(p.x_packed) for _ in range(3)]
+            self.cu_resp = torch.empty(p.B + 1, dtype=torch.int32, device=dev)
+        return self.kv_cache
+
+    def prefill_step(self, stream=None):
+        """A truncated step that also fills every layer's prefix K/V cache from
+        that layer's input (the visual + prompt rows of each packed segment)."""
+        p = self.path
+        caches = self._cache_buffers()
+        cur = p.x_packed
+        for li, w in enumerate(self.layers):
+            S.seer_kv_prefill(w.struct(), p.dims, p.dtype, cur, p.cu, self.ctx_len, p.B, p.T_full, caches[li], p.cu,
+                              p.T_full, p.ws, p.ws_bytes, stream=stream)
+            out = self.buf[li % 2] if cur is not self.buf[li % 2] else self.buf[(li + 1) % 2]
+            S.seer_layer_forward(w.struct(), p.dims, p.dtype, cur, out, p.cu, p.kv, p.B, p.T_full, None, 0, 0.0, None,
+                                 p.ws, p.ws_bytes, stream=stream)
+            cur = out
+        return cur
+
+    def cached_step(self, resp_cap=None, stream=None):
+        """A step over the response rows only: prefix keys/values come from the
+        caches (Table 7: truncation composes with prefix KV caching).  Launches
+        are sized for ``resp_cap`` response rows (default: the whole buffer);
+        the kernels read the true count from ``cu_resp[B]``.  Returns the last
+        layer's output rows in the response layout (``cu_resp``)."""
+        p = self.path
+        caches = self._cache_buffers()
+        cap = p.T_full if resp_cap is None else min(int(resp_cap), p.T_full)
+        S.seer_gather_response(p.x_packed, p.dtype, p.cu, self.ctx_len, p.B, p.dims.d_model, p.T_full, self.resp[0],
+                               self.cu_resp, stream=stream)
+        cur = self.resp[0]
+        for li, w in enumerate(self.layers):
+            out = self.resp[1] if cur is not self.resp[1] else self.resp[2]
+            S.seer_layer_forward_cached(w.struct(), p.dims, p.dtype, cur, out, self.cu_resp, self.ctx_len, p.B, cap,
+                                        caches[li], p.cu, p.kv, p.T_full, p.ws, p.ws_bytes, stream=stream)
+            cur = out
+        return cur
+
+    def cached_graph(self, resp_cap: int):
+        """Graph of one cached step sized for ``resp_cap`` response rows."""
+        cap = min(int(resp_cap), self.path.T_full)
+        self._cache_buffers()
+        return self.capture(("cached", cap), lambda stream: self.cached_step(cap, stream=stream))
 
     def truncated_graph(self, capacity: int):
         """Graph of one truncated step sized for ``capacity`` packed rows."""

@@ -22,8 +22,9 @@ SEER_F32, SEER_BF16, SEER_F16 = 0, 1, 2
 PATH_STATIC, PATH_VARLEN, PATH_EAGER = 0, 1, 2
 MAX_GROUPS = 32
 CTRL_WORDS = 8 + 4 * MAX_GROUPS
-N_PHASES = 10
-PHASES = ("detect_gemm", "snr_scan", "pack", "norm1", "qkv", "attention", "o_proj", "norm2", "gate_up", "down")
+N_PHASES = 11
+PHASES = ("detect_gemm", "snr_scan", "pack", "norm1", "qkv", "attention", "o_proj", "norm2", "gate_up", "down",
+          "kv_cache")
 
 _STATUS = {0: "SEER_OK", 1: "SEER_ERR_INVALID_ARG", 2: "SEER_ERR_UNSUPPORTED", 3: "SEER_ERR_WORKSPACE",
            4: "SEER_ERR_CUDA", 5: "SEER_ERR_TIMEOUT", 6: "SEER_ERR_DEVICE"}
@@ -71,6 +72,11 @@ def lib() -> ctypes.CDLL:
             "seer_poll_ctrl": [vp, ctypes.c_int32, i32, vp],
             "seer_sparsity_counts": [vp, i32, i32, vp, i32, i32, vp, vp, ctypes.POINTER(seer_dims), ctypes.c_float,
                                      i32, vp, vp],
+            "seer_kv_prefill": [ctypes.POINTER(seer_layer_weights), ctypes.POINTER(seer_dims), i32, vp, vp, vp, i32, i32,
+                                vp, vp, i32, vp, sz, vp],
+            "seer_layer_forward_cached": [ctypes.POINTER(seer_layer_weights), ctypes.POINTER(seer_dims), i32, vp, vp,
+                                          vp, vp, i32, i32, vp, vp, vp, i32, vp, sz, vp],
+            "seer_gather_response": [vp, i32, vp, vp, i32, i32, i32, vp, vp, vp],
             "seer_snr_scan": [vp, i32, i32, i32, ctypes.POINTER(seer_params), vp, vp, vp],
             "seer_layer_forward": [ctypes.POINTER(seer_layer_weights), ctypes.POINTER(seer_dims), i32, vp, vp, vp, vp,
                                    i32, i32, vp, i32, ctypes.c_float, vp, vp, sz, vp],
@@ -164,6 +170,23 @@ def seer_sparsity_counts(x, dt, T_rows, resp_start, B, N, w_gate, w_up, dims, ac
     _check(lib().seer_sparsity_counts(_p(x), _dt(dt), T_rows, _p(resp_start), B, N, _p(w_gate), _p(w_up),
                                       ctypes.byref(dims), act_eps, 1 if accumulate else 0, _p(counts_inout),
                                       _stream(stream)))
+
+
+def seer_kv_prefill(w, dims, dt, x, cu_x, ctx_len, B, T_x_cap, kv_cache, cu_kv, T_kv_cap, ws, ws_bytes, stream=None):
+    _check(lib().seer_kv_prefill(ctypes.byref(w), ctypes.byref(dims), _dt(dt), _p(x), _p(cu_x), _p(ctx_len), B, T_x_cap,
+                                 _p(kv_cache), _p(cu_kv), T_kv_cap, _p(ws), ws_bytes, _stream(stream)))
+
+
+def seer_layer_forward_cached(w, dims, dt, x_resp, y_resp, cu_resp, ctx_len, B, T_resp_cap, kv_cache, cu_kv, kv_len,
+                              T_kv_cap, ws, ws_bytes, stream=None):
+    _check(lib().seer_layer_forward_cached(ctypes.byref(w), ctypes.byref(dims), _dt(dt), _p(x_resp), _p(y_resp),
+                                           _p(cu_resp), _p(ctx_len), B, T_resp_cap, _p(kv_cache), _p(cu_kv),
+                                           _p(kv_len), T_kv_cap, _p(ws), ws_bytes, _stream(stream)))
+
+
+def seer_gather_response(x_packed, dt, cu, ctx_len, B, d, T_cap, x_resp, cu_resp_out, stream=None):
+    _check(lib().seer_gather_response(_p(x_packed), _dt(dt), _p(cu), _p(ctx_len), B, d, T_cap, _p(x_resp),
+                                      _p(cu_resp_out), _stream(stream)))
 
 
 def seer_snr_scan(counts, B, N, F, params, L_star_out, i_star_out=None, stream=None):

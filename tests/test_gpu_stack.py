@@ -187,3 +187,19 @@ def test_step0_truncated_after_detection_layer(st):
     rows = sorted({0, int(seg[b]) - 1, int(st["lens"].ctx[b]), *map(int, rng.integers(0, int(seg[b]), 20))})
     ref = oracle.layer_forward_rows(hp[cu[b]:cu[b + 1]], w, wl.n_heads, rows, kv_len=int(kv[b]))
     check_close(y[cu[b] + np.asarray(rows)], ref, "bf16", "step-0 layer after detection")
+
+
+def test_stack_cached_step_equals_truncated_step(st):
+    # Table 7 composition: with the prefix K/V cached from the same step input, a
+    # step over the response rows only reproduces the truncated step's rows exactly
+    stack = st["stack"]
+    p = stack.path
+    full = stack.prefill_step().clone()
+    out = stack.cached_step()
+    torch.cuda.synchronize()
+    cu, c = p.cu.cpu().numpy(), st["lens"].ctx
+    cr = stack.cu_resp.cpu().numpy()
+    np.testing.assert_array_equal(cr, cu - np.concatenate([[0], np.cumsum(c)]))
+    a, f = host(out), host(full)
+    for b in range(st["wl"].batch):
+        np.testing.assert_array_equal(a[cr[b]:cr[b + 1]], f[cu[b] + c[b]:cu[b + 1]])
