@@ -120,9 +120,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int b = wk.x, h = wk.y, qt0 = wk.z, nt = wk.w;   // query tiles qt0 .. qt0 + nt - 1
   const int seq0 = p.cu[b];
   const int L = p.cu[b + 1] - seq0;
-  const int kvL = p.kv_len ? p.kv_len[b] : L;
-  const int q0 = seq0 + qt0 * BQ;
   const int kv0 = p.cu_kv ? p.cu_kv[b] : seq0;  // first K/V row of the segment
+  const int kvL = p.kv_len ? p.kv_len[b] : (p.cu_kv ? p.cu_kv[b + 1] - kv0 : L);
+  const int q0 = seq0 + qt0 * BQ;
   const int nkv = (kvL + BKV - 1) / BKV;
   const int xq = h * DH, xk = p.xk0 + h * DH, xv = p.xv0 + h * DH;
 
