@@ -247,6 +247,14 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi, bool f16) { return
 __device__ __forceinline__ float lo16(uint32_t v, bool f16) { return f16 ? f16_lo(v) : bf16_lo(v); }
 __device__ __forceinline__ float hi16(uint32_t v, bool f16) { return f16 ? f16_hi(v) : bf16_hi(v); }
 
+// 32-byte global store (one full sector); p must be 32-byte aligned.
+__device__ __forceinline__ void st_global_v8(void* p, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t a4,
+                                             uint32_t a5, uint32_t a6, uint32_t a7) {
+  asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(a0), "r"(a1), "r"(a2), "r"(a3),
+               "r"(a4), "r"(a5), "r"(a6), "r"(a7)
+               : "memory");
+}
+
 // Element storage types understood by the element-wise kernels.
 enum ElemType : int { kF32 = 0, kBF16 = 1, kF16 = 2 };
 

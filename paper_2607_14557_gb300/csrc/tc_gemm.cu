@@ -243,14 +243,16 @@ __global__ void __launch_bounds__(THREADS, 1)
                 v0[e] = fmaf(x0, cs[e], -x1 * sn[e]);
                 v1[e] = fmaf(x1, cs[e], x0 * sn[e]);
               }
-              uint4* p0 = reinterpret_cast<uint4*>(crow + c0);
-              uint4* p1 = reinterpret_cast<uint4*>(crow + c1);
 #pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                p0[i] = make_uint4(pack2(v0[8 * i + 0], v0[8 * i + 1], of16), pack2(v0[8 * i + 2], v0[8 * i + 3], of16),
-                                   pack2(v0[8 * i + 4], v0[8 * i + 5], of16), pack2(v0[8 * i + 6], v0[8 * i + 7], of16));
-                p1[i] = make_uint4(pack2(v1[8 * i + 0], v1[8 * i + 1], of16), pack2(v1[8 * i + 2], v1[8 * i + 3], of16),
-                                   pack2(v1[8 * i + 4], v1[8 * i + 5], of16), pack2(v1[8 * i + 6], v1[8 * i + 7], of16));
+              for (int i = 0; i < 2; ++i) {
+                const float* w0 = v0 + 16 * i;
+                const float* w1 = v1 + 16 * i;
+                st_global_v8(crow + c0 + 16 * i, pack2(w0[0], w0[1], of16), pack2(w0[2], w0[3], of16),
+                             pack2(w0[4], w0[5], of16), pack2(w0[6], w0[7], of16), pack2(w0[8], w0[9], of16),
+                             pack2(w0[10], w0[11], of16), pack2(w0[12], w0[13], of16), pack2(w0[14], w0[15], of16));
+                st_global_v8(crow + c1 + 16 * i, pack2(w1[0], w1[1], of16), pack2(w1[2], w1[3], of16),
+                             pack2(w1[4], w1[5], of16), pack2(w1[6], w1[7], of16), pack2(w1[8], w1[9], of16),
+                             pack2(w1[10], w1[11], of16), pack2(w1[12], w1[13], of16), pack2(w1[14], w1[15], of16));
               }
             }
           }
@@ -283,11 +285,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                 v[8 * i + 6] += lo16(rv.w, rf16); v[8 * i + 7] += hi16(rv.w, rf16);
               }
             }
-            uint4* cp = reinterpret_cast<uint4*>(crow + c * 32);
+            // a lane owns one row: 64 contiguous bytes per chunk as two full 32-byte sectors
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              cp[i] = make_uint4(pack2(v[8 * i + 0], v[8 * i + 1], of16), pack2(v[8 * i + 2], v[8 * i + 3], of16),
-                                 pack2(v[8 * i + 4], v[8 * i + 5], of16), pack2(v[8 * i + 6], v[8 * i + 7], of16));
+            for (int i = 0; i < 2; ++i) {
+              const float* w = v + 16 * i;
+              st_global_v8(crow + c * 32 + 16 * i, pack2(w[0], w[1], of16), pack2(w[2], w[3], of16),
+                           pack2(w[4], w[5], of16), pack2(w[6], w[7], of16), pack2(w[8], w[9], of16),
+                           pack2(w[10], w[11], of16), pack2(w[12], w[13], of16), pack2(w[14], w[15], of16));
             }
           }
         }
@@ -332,11 +336,12 @@ __global__ void __launch_bounds__(THREADS, 1)
             cnt += fabsf(a[i]) < p.act_eps ? 1 : 0;
           }
           if (MODE == kGemmSwiglu && store) {
-            uint4* cp = reinterpret_cast<uint4*>(arow + c * 32);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              cp[i] = make_uint4(pack2(a[8 * i + 0], a[8 * i + 1], of16), pack2(a[8 * i + 2], a[8 * i + 3], of16),
-                                 pack2(a[8 * i + 4], a[8 * i + 5], of16), pack2(a[8 * i + 6], a[8 * i + 7], of16));
+            for (int i = 0; i < 2; ++i) {
+              const float* w = a + 16 * i;
+              st_global_v8(arow + c * 32 + 16 * i, pack2(w[0], w[1], of16), pack2(w[2], w[3], of16),
+                           pack2(w[4], w[5], of16), pack2(w[6], w[7], of16), pack2(w[8], w[9], of16),
+                           pack2(w[10], w[11], of16), pack2(w[12], w[13], of16), pack2(w[14], w[15], of16));
             }
           }
         }
