@@ -65,8 +65,10 @@ int tc_gemm_smem_bytes();
 // L2 raster of the persistent GEMM (GemmParams::group_m) for a B operand of
 // b_bytes and an A row-tile of a_tile_bytes.
 int tc_gemm_group_m(long b_bytes, long a_tile_bytes);
+// mC: the 16-bit output C (Store, Residual, Rope) or act (Swiglu) with 32 x 32
+// boxes and no swizzle, for the epilogue's TMA stores (unused by Count).
 cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
-                           const GemmParams& p, int num_sms, cudaStream_t st);
+                           const CUtensorMap& mC, const GemmParams& p, int num_sms, cudaStream_t st);
 int tc_attn_smem_bytes();
 cudaError_t launch_tc_attn(const CUtensorMap& mQ, const CUtensorMap& mKV, const AttnParams& p, int grid, bool f16,
                            cudaStream_t st);

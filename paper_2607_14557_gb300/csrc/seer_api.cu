@@ -96,7 +96,7 @@ std::once_flag g_encode_once;
 // Row-major [rows, cols] 16-bit matrix with leading dimension ld elements,
 // boxes of 64 columns (128 bytes, 128-byte swizzle) x box_rows rows.
 seer_status make_map16(CUtensorMap* m, const void* base, seer_dtype dt, uint64_t rows, uint64_t cols, uint64_t ld,
-                       uint32_t box_rows) {
+                       uint32_t box_rows, uint32_t box_cols = 64, bool swizzle128 = true) {
   std::call_once(g_encode_once, [] {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -107,11 +107,12 @@ seer_status make_map16(CUtensorMap* m, const void* base, seer_dtype dt, uint64_t
   if (g_encode == nullptr) return fail(SEER_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
   cuuint64_t dims[2] = {cols, rows > 0 ? rows : 1};
   cuuint64_t strides[1] = {ld * 2};
-  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
   const CUtensorMapDataType ty = dt == SEER_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   CUresult r = g_encode(m, ty, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                        swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(SEER_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
   return SEER_OK;
 }
@@ -263,11 +264,12 @@ seer_status do_linear(const void* a, const void* w, seer_dtype op_dt, const void
     if (M_cap == 0) return SEER_OK;
     p.idesc = make_idesc(128, 256, 0, op_dt == SEER_F16);
     p.group_m = tc_gemm_group_m(2l * N * K, 2l * 128 * K);
-    CUtensorMap mA, mB;
+    CUtensorMap mA, mB, mC;
     SEER_TRY(make_map16(&mA, a, op_dt, M_cap, K, K, 128));
     SEER_TRY(make_map16(&mB, w, op_dt, N, K, K, 128));
+    SEER_TRY(make_map16(&mC, c, c_dt, M_cap, N, N, 32, 32, false));
     Phase ph(phase, st);
-    SEER_CUDA(launch_tc_gemm(mode, mA, mB, mB, p, di->num_sms, st), "tc_gemm launch");
+    SEER_CUDA(launch_tc_gemm(mode, mA, mB, mB, mC, p, di->num_sms, st), "tc_gemm launch");
   } else {
     if (c_dt != SEER_F32 || (r && r_dt != SEER_F32)) return fail(SEER_ERR_UNSUPPORTED, "fp32 linear needs fp32 output");
     if (M_cap == 0) return SEER_OK;
@@ -326,12 +328,14 @@ seer_status do_swiglu(const void* a, const void* wg, const void* wu, seer_dtype 
   if (is16(op_dt)) {
     p.idesc = make_idesc(128, 256, 0, op_dt == SEER_F16);
     p.group_m = tc_gemm_group_m(2l * 2 * F * K, 2l * 128 * K);
-    CUtensorMap mA, mG, mU;
+    CUtensorMap mA, mG, mU, mC;
     SEER_TRY(make_map16(&mA, a, op_dt, M_cap, K, K, 128));
     SEER_TRY(make_map16(&mG, wg, op_dt, F, K, K, 128));
     SEER_TRY(make_map16(&mU, wu, op_dt, F, K, K, 128));
+    if (mode == kGemmSwiglu) SEER_TRY(make_map16(&mC, act, act_dt, M_cap, F, F, 32, 32, false));
+    else mC = mA;                                  // Count stores nothing
     Phase ph(phase, st);
-    SEER_CUDA(launch_tc_gemm(mode, mA, mG, mU, p, di->num_sms, st), "tc_gemm launch");
+    SEER_CUDA(launch_tc_gemm(mode, mA, mG, mU, mC, p, di->num_sms, st), "tc_gemm launch");
   } else {
     Phase ph(phase, st);
     SEER_CUDA(launch_simt_gemm(mode, static_cast<const float*>(a), static_cast<const float*>(wg),

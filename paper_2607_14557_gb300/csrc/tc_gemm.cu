@@ -11,7 +11,9 @@
 //               256-column fp32 accumulators (double buffered, 512 columns);
 //   warps 2-5   epilogue: tcgen05.ld of the accumulator (each warp owns one
 //               32-lane quarter of TMEM = 32 output rows), fused epilogue,
-//               16-byte global stores.
+//               32 x 32 output chunks staged in shared memory and written by
+//               TMA stores marked L2 evict-first (a tile whose rows run past
+//               the device row count stores its valid rows lane by lane).
 // The epilogue of tile t overlaps the main loop of tile t+1.
 //
 // Epilogues (Sec. 3.1 Eq. 2 projections; Sec. 3.2 sparsity hook):
@@ -41,7 +43,9 @@ constexpr int TMEM_COLS = 512;
 constexpr int BAR_BYTES = 256;
 constexpr int ROPE_HEAD = 128;                       // head width of the Rope epilogue
 constexpr int ROPE_BYTES = ROPE_HEAD / 2 * 8;        // (hi, lo) inverse frequency per pair
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + ROPE_BYTES + 1024;
+constexpr int EPI_CHUNK = 32 * 32 * 2;              // a warp's 32 rows x 32 columns, 16-bit
+constexpr int EPI_BYTES = 4 * 2 * EPI_CHUNK;         // 4 epilogue warps x 2 staging buffers
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + ROPE_BYTES + EPI_BYTES + 1024;
 
 // Raster: groups of `group_m` m-tiles; inside a group m varies fastest and
 // the group sweeps every n-tile.  group_m = 1 keeps the whole B operand hot in
@@ -62,7 +66,7 @@ __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)
 template <int MODE>
 __global__ void __launch_bounds__(THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB0,
-                   const __grid_constant__ CUtensorMap mB1, const GemmParams p) {
+                   const __grid_constant__ CUtensorMap mB1, const __grid_constant__ CUtensorMap mC, const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
@@ -72,6 +76,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float2* rope_tab = reinterpret_cast<float2*>(smem + STAGES * STAGE_BYTES + BAR_BYTES);
+  uint8_t* epi_stage = smem + STAGES * STAGE_BYTES + BAR_BYTES + ROPE_BYTES;   // [4 warps][2][EPI_CHUNK]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -199,6 +204,28 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int q = warp & 3;                    // TMEM lane quarter owned by this warp
     const int row_in_tile = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    uint8_t* my_stage = epi_stage + q * 2 * EPI_CHUNK;
+    // outputs stream through L2 marked evict-first, so they do not push the
+    // operand slabs the raster keeps resident out of the cache
+    const uint64_t out_policy = l2_policy_evict_first();
+    int n_chunks = 0;                            // bulk stores issued by this warp (staging buffer = n & 1)
+    // one staged 32 x 32 chunk of this warp's rows -> a TMA store at (x, y); the
+    // buffer used two chunks ago is reused only once its store has read it
+    auto store_chunk = [&](const uint32_t (&w)[16], int x, int y) {
+      uint8_t* buf = my_stage + (n_chunks & 1) * EPI_CHUNK;
+      if (lane == 0 && n_chunks >= 2) bulk_wait_read_1();
+      __syncwarp();
+      uint4* d = reinterpret_cast<uint4*>(buf + lane * 64);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) d[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d_hint(&mC, buf, x, y, out_policy);
+        bulk_commit();
+      }
+      ++n_chunks;
+    };
     if (MODE == kGemmRope) {
       const int et = threadIdx.x - 64;                 // 0..127 over the epilogue warps
       if (et < ROPE_HEAD / 2) rope_tab[et] = rope_inv_freq(et, ROPE_HEAD, p.rope_theta);
@@ -260,6 +287,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       } else if (MODE == kGemmStore || MODE == kGemmResidual) {
         const int row = m * BM + row_in_tile;
         const bool valid = row < M;
+        const bool slab_full = m * BM + q * 32 + 32 <= M;      // this warp's 32 rows all valid: TMA store
         const bool of16 = p.out_type == kF16, rf16 = p.res_type == kF16;
         uint16_t* crow = reinterpret_cast<uint16_t*>(p.C) + static_cast<size_t>(valid ? row : 0) * p.ldc + n * BN;
         const uint16_t* rrow =
@@ -270,7 +298,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint32_t r[32];
           tmem_ld32(tacc + c * 32, r);
           tmem_ld_wait();
-          if (valid) {
+          if (slab_full || valid) {
             float v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
@@ -285,13 +313,15 @@ __global__ void __launch_bounds__(THREADS, 1)
                 v[8 * i + 6] += lo16(rv.w, rf16); v[8 * i + 7] += hi16(rv.w, rf16);
               }
             }
-            // a lane owns one row: 64 contiguous bytes per chunk as two full 32-byte sectors
+            uint32_t w[16];
 #pragma unroll
-            for (int i = 0; i < 2; ++i) {
-              const float* w = v + 16 * i;
-              st_global_v8(crow + c * 32 + 16 * i, pack2(w[0], w[1], of16), pack2(w[2], w[3], of16),
-                           pack2(w[4], w[5], of16), pack2(w[6], w[7], of16), pack2(w[8], w[9], of16),
-                           pack2(w[10], w[11], of16), pack2(w[12], w[13], of16), pack2(w[14], w[15], of16));
+            for (int i = 0; i < 16; ++i) w[i] = pack2(v[2 * i], v[2 * i + 1], of16);
+            if (slab_full) {
+              store_chunk(w, n * BN + c * 32, m * BM + q * 32);
+            } else {
+              // a lane owns one row: 64 contiguous bytes as two full 32-byte sectors
+              st_global_v8(crow + c * 32, w[0], w[1], w[2], w[3], w[4], w[5], w[6], w[7]);
+              st_global_v8(crow + c * 32 + 16, w[8], w[9], w[10], w[11], w[12], w[13], w[14], w[15]);
             }
           }
         }
@@ -335,13 +365,18 @@ __global__ void __launch_bounds__(THREADS, 1)
             a[i] = silu_f(__uint_as_float(g[i])) * __uint_as_float(u[i]);
             cnt += fabsf(a[i]) < p.act_eps ? 1 : 0;
           }
-          if (MODE == kGemmSwiglu && store) {
+          if (MODE == kGemmSwiglu) {
+            const bool slab_full = m * BM + q * 32 + 32 <= M;
+            if (slab_full || store) {
+              uint32_t w[16];
 #pragma unroll
-            for (int i = 0; i < 2; ++i) {
-              const float* w = a + 16 * i;
-              st_global_v8(arow + c * 32 + 16 * i, pack2(w[0], w[1], of16), pack2(w[2], w[3], of16),
-                           pack2(w[4], w[5], of16), pack2(w[6], w[7], of16), pack2(w[8], w[9], of16),
-                           pack2(w[10], w[11], of16), pack2(w[12], w[13], of16), pack2(w[14], w[15], of16));
+              for (int i = 0; i < 16; ++i) w[i] = pack2(a[2 * i], a[2 * i + 1], of16);
+              if (slab_full) {
+                store_chunk(w, n * 128 + c * 32, m * BM + q * 32);
+              } else {
+                st_global_v8(arow + c * 32, w[0], w[1], w[2], w[3], w[4], w[5], w[6], w[7]);
+                st_global_v8(arow + c * 32 + 16, w[8], w[9], w[10], w[11], w[12], w[13], w[14], w[15]);
+              }
             }
           }
         }
@@ -352,6 +387,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (lane == 0) mbar_arrive(&acc_empty[acc]);
       if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
     }
+    if (lane == 0) bulk_wait_all();              // outputs written before the CTA exits
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -363,8 +400,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 }
 
 template <int MODE>
-cudaError_t launch_mode(const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1, const GemmParams& p,
-                        int num_sms, cudaStream_t st) {
+cudaError_t launch_mode(const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1, const CUtensorMap& mC,
+                        const GemmParams& p, int num_sms, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
@@ -378,7 +415,7 @@ cudaError_t launch_mode(const CUtensorMap& mA, const CUtensorMap& mB0, const CUt
   long tiles = num_m * num_n;
   if (tiles <= 0) return cudaSuccess;
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  tc_gemm_kernel<MODE><<<grid, THREADS, SMEM_BYTES, st>>>(mA, mB0, mB1, p);
+  tc_gemm_kernel<MODE><<<grid, THREADS, SMEM_BYTES, st>>>(mA, mB0, mB1, mC, p);
   return cudaGetLastError();
 }
 
@@ -400,13 +437,13 @@ int tc_gemm_group_m(long b_bytes, long a_tile_bytes) {
 }
 
 cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
-                           const GemmParams& p, int num_sms, cudaStream_t st) {
+                           const CUtensorMap& mC, const GemmParams& p, int num_sms, cudaStream_t st) {
   switch (mode) {
-    case kGemmStore: return launch_mode<kGemmStore>(mA, mB0, mB1, p, num_sms, st);
-    case kGemmResidual: return launch_mode<kGemmResidual>(mA, mB0, mB1, p, num_sms, st);
-    case kGemmSwiglu: return launch_mode<kGemmSwiglu>(mA, mB0, mB1, p, num_sms, st);
-    case kGemmCount: return launch_mode<kGemmCount>(mA, mB0, mB1, p, num_sms, st);
-    case kGemmRope: return launch_mode<kGemmRope>(mA, mB0, mB1, p, num_sms, st);
+    case kGemmStore: return launch_mode<kGemmStore>(mA, mB0, mB1, mC, p, num_sms, st);
+    case kGemmResidual: return launch_mode<kGemmResidual>(mA, mB0, mB1, mC, p, num_sms, st);
+    case kGemmSwiglu: return launch_mode<kGemmSwiglu>(mA, mB0, mB1, mC, p, num_sms, st);
+    case kGemmCount: return launch_mode<kGemmCount>(mA, mB0, mB1, mC, p, num_sms, st);
+    case kGemmRope: return launch_mode<kGemmRope>(mA, mB0, mB1, mC, p, num_sms, st);
     default: return cudaErrorInvalidValue;
   }
 }
