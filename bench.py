@@ -335,6 +335,11 @@ def run_stack(args, wl, world, rank, local):
                         + (nl * 8 + 3) + nl * 13 + (n_steps - 2) * (2 + nl * 9), "clocks": clk.summary(),
         "peak_source": src,
     }
+    if world == 1 and rank == 0 and not args.no_cpu_baseline:
+        k, dt, sample = oracle_sample(wl)
+        line["cpu_baseline"] = {"value": k / dt, "unit": "tokens/s (token-layers: one layer pass)",
+                                "cores": len(os.sched_getaffinity(0)), "kind": "oracle", "sample": sample,
+                                "seconds": dt}
     if rank == 0:
         print(json.dumps(line), flush=True)
 
