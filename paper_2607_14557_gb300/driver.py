@@ -144,6 +144,61 @@ class SeerPath:
         self.pack(x_full, cu_full, ctx_len, stream)
         self.layer(w, stream=stream)
 
+    def run_from_host(self, x_host, cu_full, resp_start, ctx_len, w: LayerWeights, y_host, L_host, steps: int,
+                      stream=None, copy_stream=None) -> Dict[str, object]:
+        """``steps`` end-to-end steps from pinned host memory: every step copies
+        its full-window input host -> device, runs detect -> route/pack ->
+        truncated layer, and copies the packed output rows and L* device ->
+        host.  Copies run on ``copy_stream`` with double-buffered device
+        inputs and outputs, so step i+1's upload and step i-1's download
+        overlap step i's compute.  Returns the route of the last step; all
+        copies have completed on return."""
+        dev = self.device
+        stream = stream or torch.cuda.current_stream(dev)
+        copy_stream = copy_stream or torch.cuda.Stream(dev)
+        if getattr(self, "_x_in", None) is None or self._x_in[0].shape != x_host.shape:
+            self._x_in = [torch.empty(x_host.shape, dtype=x_host.dtype, device=dev) for _ in range(2)]
+            self._y_out = [self.y, torch.empty_like(self.y)]
+            self._L_out = [torch.empty_like(self.L_star) for _ in range(2)]
+        x_in, y_out, L_out = self._x_in, self._y_out, self._L_out
+        loaded = [torch.cuda.Event() for _ in range(2)]      # input buffer holds its step's data
+        consumed = [torch.cuda.Event() for _ in range(2)]    # compute no longer reads the input buffer
+        computed = [torch.cuda.Event() for _ in range(2)]    # output buffer holds its step's result
+        drained = [torch.cuda.Event() for _ in range(2)]     # output buffer copied to the host
+        for e in consumed + drained:
+            e.record(stream)
+
+        def upload(i):
+            b = i % 2
+            copy_stream.wait_event(consumed[b])
+            with torch.cuda.stream(copy_stream):
+                x_in[b].copy_(x_host, non_blocking=True)
+            loaded[b].record(copy_stream)
+
+        route = None
+        upload(0)
+        for i in range(steps):
+            b = i % 2
+            if i + 1 < steps:
+                upload(i + 1)
+            stream.wait_event(loaded[b])
+            stream.wait_event(drained[b])
+            self.detect(x_in[b], resp_start, w, stream)
+            self.pack(x_in[b], cu_full, ctx_len, stream)
+            consumed[b].record(stream)
+            self.layer(w, y=y_out[b], stream=stream)
+            L_out[b].copy_(self.L_star, non_blocking=True)
+            computed[b].record(stream)
+            route = self.route()                 # host learns the packed total while the layer runs
+            copy_stream.wait_event(computed[b])
+            with torch.cuda.stream(copy_stream):
+                y_host[:route["total"]].copy_(y_out[b][:route["total"]], non_blocking=True)
+                L_host.copy_(L_out[b], non_blocking=True)
+            drained[b].record(copy_stream)
+        copy_stream.synchronize()
+        stream.synchronize()
+        return route
+
     def route(self, timeout_us: int = 10_000_000) -> Dict[str, object]:
         """Read the route of the last pack from the pinned control word."""
         S.seer_poll_ctrl(self.host_ctrl, self.epoch, timeout_us, self.ctrl)

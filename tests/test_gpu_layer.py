@@ -210,3 +210,31 @@ def test_rotary_layer_at_long_positions():
         rows = sorted({0, 1, L - 1, L - 2, *map(int, rng.integers(L // 2, L, 14))})
         ref = oracle.layer_forward_rows(x[cu_full[b]:cu_full[b + 1]], w, wl.n_heads, rows, rope_theta=1e4)
         check_close(yh[cu_full[b] + np.asarray(rows)], ref, "bf16", f"rotary layer segment {b}")
+
+
+def test_run_from_host_pipelined_matches_device_step():
+    # the end-to-end call (pinned host input, double-buffered copies overlapping compute)
+    # returns exactly what a device-resident step computes
+    from paper_2607_14557_gb300 import driver as D
+    wl = synth.tiny_workload(dtype="bf16", seed=390, d=256, n_heads=2, head_dim=128, d_ff=768, batch=3, window=160,
+                             boundary=("uniform", 8, 150))
+    lens = synth.lengths(wl)
+    x, cu_full, resp = synth.hidden_full(wl, lens)
+    w = synth.layer_weights(wl, 0)
+    dims = S.make_dims(wl.d, wl.n_heads, wl.head_dim, wl.d_ff)
+    W = D.LayerWeights.from_host(w, "bf16")
+    path = D.SeerPath(dims, "bf16", wl.batch, wl.window, x.shape[0], S.make_params(wl.act_eps))
+    cuf, rs, ctx = i32(cu_full), i32(resp), i32(lens.ctx)
+    xd = to_dev(x, "bf16")
+    path.step(xd, cuf, rs, ctx, W)
+    torch.cuda.synchronize()
+    T = int(path.cu[-1].item())
+    ref = host(path.y)[:T]
+    x_host = xd.cpu().pin_memory()
+    y_host = torch.full((x.shape[0], wl.d), 7.0, dtype=torch.bfloat16).pin_memory()
+    L_host = torch.zeros(wl.batch, dtype=torch.int32).pin_memory()
+    r = path.run_from_host(x_host, cuf, rs, ctx, W, y_host, L_host, 3)
+    assert r["total"] == T
+    np.testing.assert_array_equal(y_host.float().numpy()[:T], ref)
+    assert (y_host.float().numpy()[T:] == 7.0).all()
+    np.testing.assert_array_equal(L_host.numpy(), lens.boundary + 1)
