@@ -33,6 +33,7 @@ if ROOT not in sys.path:
 
 import synth  # noqa: E402
 
+PRECISION = "bf16 layer inputs/outputs, f16 tensor-core operands and intermediates, fp32 accumulation"
 METRIC = "truncated denoise-layer tokens/s & TFLOP/s vs BF16 peak; speedup over padded"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 KERNELS_PER_STEP = 11   # detect GEMM, scan, pack, norm, QKV, attn schedule, attn, O proj, norm, gate/up, down
@@ -305,7 +306,7 @@ def run_stack(args, wl, world, rank, local):
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": n_steps,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_seer / n_steps, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16 in/out, f16 tensor-core operands, f32 accumulate", "data": "synthetic",
+        "vs_baseline": None, "dtype": "f16", "precision": PRECISION, "data": "synthetic",
         "config": {"workload": f"{wl.name} (workload 3): {nl} layers x {n_steps} denoising steps, batch {wl.batch}, "
                                f"window {wl.window}, d {d}, F {F}; tokens counted once per layer and step",
                    "tokens_full": T_full, "tokens_valid": T_valid, "tokens_executed": T_exec, "L_star": L.tolist(),
@@ -369,24 +370,16 @@ def main():
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
 
+    from paper_2607_14557_gb300 import replicas as R
+
     def barrier():
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
+        R.barrier(dev)
 
     def max_over_ranks(v):
-        if world == 1:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return R.max_over_ranks(v, dev)
 
     def sum_over_ranks(v):
-        if world == 1:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        return float(t.item())
+        return R.sum_over_ranks(v, dev)
 
     # ---- synthetic inputs, resident in HBM before timing
     lens = synth.lengths(wl)
@@ -527,7 +520,8 @@ def main():
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step_max, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16 in/out, f16 tensor-core operands, f32 accumulate" if wl.dtype == "bf16" else "f32",
+        "vs_baseline": None, "dtype": "f16" if wl.dtype == "bf16" else "f32",
+        "precision": PRECISION if wl.dtype == "bf16" else "fp32 storage and arithmetic (CUDA cores)",
         "data": "synthetic",
         "config": {"workload": f"{wl.name} (workload {wl.index}): batch {wl.batch}, window {wl.window}, "
                                f"d {wl.d}, heads {wl.n_heads}x{wl.head_dim}, F {wl.d_ff}",
