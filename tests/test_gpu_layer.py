@@ -238,3 +238,44 @@ def test_run_from_host_pipelined_matches_device_step():
     np.testing.assert_array_equal(y_host.float().numpy()[:T], ref)
     assert (y_host.float().numpy()[T:] == 7.0).all()
     np.testing.assert_array_equal(L_host.numpy(), lens.boundary + 1)
+
+
+def test_tiny_f16_model_path():
+    # an f16 model (inputs, weights and outputs f16) through detect -> pack -> layer
+    wl = synth.tiny_workload(dtype="bf16", seed=395, d=256, n_heads=2, head_dim=128, d_ff=768, batch=3, window=160,
+                             boundary=("uniform", 8, 150))
+    lens = synth.lengths(wl)
+    xb, cu_full, resp = synth.hidden_full(wl, lens)
+    wb = synth.layer_weights(wl, 0)
+    f16 = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float32)).to(torch.float16)
+    x = f16(xb).double().numpy()
+    w = {k: f16(v).double().numpy() for k, v in wb.items()}
+    B, N, F, d = wl.batch, wl.window, wl.d_ff, wl.d
+    dims = S.make_dims(d, wl.n_heads, wl.head_dim, F)
+    params = S.make_params(wl.act_eps)
+    dev = lambda a: f16(a).to(cuda())
+    Wt = {"w_qkv": dev(np.concatenate([w["wq"], w["wk"], w["wv"]])), "w_o": dev(w["wo"]), "w_gate": dev(w["wg"]),
+          "w_up": dev(w["wu"]), "w_down": dev(w["wd"]), "g_attn": dev(w["g_attn"]), "g_mlp": dev(w["g_mlp"])}
+    xd = dev(x)
+    counts = torch.empty(B * N, dtype=torch.int32, device=cuda())
+    L = torch.empty(B, dtype=torch.int32, device=cuda())
+    S.seer_detect_boundary(xd, "f16", x.shape[0], i32(resp), B, N, Wt["w_gate"], Wt["w_up"], dims, params, counts, L)
+    T_cap = x.shape[0]
+    xp = torch.zeros((T_cap, d), dtype=torch.float16, device=cuda())
+    cu = torch.empty(B + 1, dtype=torch.int32, device=cuda())
+    kv = torch.empty(B, dtype=torch.int32, device=cuda())
+    meta = torch.empty(S.CTRL_WORDS, dtype=torch.int32, device=cuda())
+    S.seer_pack_ragged(xd, "f16", i32(cu_full), i32(lens.ctx), L, B, d, N, T_cap, params, xp, cu, kv, meta)
+    y = torch.full((T_cap, d), 9.0, dtype=torch.float16, device=cuda())
+    ws_bytes = S.seer_layer_workspace_size(dims, "f16", T_cap, B)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=cuda())
+    S.seer_layer_forward(weights_struct(Wt), dims, "f16", xp, y, cu, kv, B, T_cap, None, 0, 0.0, None, ws, ws_bytes)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(L.cpu().numpy(), lens.boundary + 1)
+    seg, kv_ref, cu_ref = oracle.segment_layout(lens.ctx, L.cpu().numpy(), N)
+    np.testing.assert_array_equal(cu.cpu().numpy(), cu_ref)
+    T = int(cu_ref[-1])
+    np.testing.assert_array_equal(host(xp)[:T], oracle.pack_rows(x, cu_full, seg))
+    ref = oracle.layer_forward_packed(host(xp)[:T], cu_ref, w, wl.n_heads, kv_len=kv_ref)
+    check_close(host(y)[:T], ref, "bf16", "f16 model layer")
+    assert (host(y)[T:] == 9.0).all()
