@@ -131,9 +131,10 @@ def snr_boundaries(counts2d, F: int, tau_jump: float = 0.03, gamma: float = 0.6,
 PATH_STATIC, PATH_VARLEN, PATH_EAGER = 0, 1, 2
 
 
-def bucket_set(n_max: int) -> List[int]:
-    """Static micro-buckets {8, 16, 32, ..., N_max} (Sec. 3.4)."""
-    out, b = [], 8
+def bucket_set(n_max: int, b_min: int = 8) -> List[int]:
+    """Static micro-buckets {8, 16, 32, ..., N_max} (Sec. 3.4); ``b_min`` is
+    the smallest bucket (the paper's set starts at 8), each next one doubles."""
+    out, b = [], int(b_min)
     while b < n_max:
         out.append(b)
         b *= 2
@@ -141,8 +142,8 @@ def bucket_set(n_max: int) -> List[int]:
     return out
 
 
-def bucket_of(L: int, n_max: int) -> int:
-    for b in bucket_set(n_max):
+def bucket_of(L: int, n_max: int, b_min: int = 8) -> int:
+    for b in bucket_set(n_max, b_min):
         if L <= b:
             return b
     raise ValueError(f"L*={L} exceeds the window {n_max}")
@@ -153,7 +154,7 @@ def padding_waste_ratio(L_stars: Sequence[int], B_G: int) -> float:
     return 1.0 - float(sum(int(v) for v in L_stars)) / float(len(L_stars) * B_G)
 
 
-def route(L_star: Sequence[int], n_max: int, tau_pad: float = 0.2, eager_max_bucket: int = 4):
+def route(L_star: Sequence[int], n_max: int, tau_pad: float = 0.2, eager_max_bucket: int = 4, bucket_min: int = 8):
     """Group sequences by micro-bucket and pick each group's path (Sec. 3.4).
 
     Returns a list of dicts (ascending bucket) with keys ``bucket``,
@@ -162,7 +163,7 @@ def route(L_star: Sequence[int], n_max: int, tau_pad: float = 0.2, eager_max_buc
     """
     groups: Dict[int, List[int]] = {}
     for i, L in enumerate(L_star):
-        groups.setdefault(bucket_of(int(L), n_max), []).append(i)
+        groups.setdefault(bucket_of(int(L), n_max, bucket_min), []).append(i)
     out = []
     for b in sorted(groups):
         mem = groups[b]
@@ -180,7 +181,7 @@ def route(L_star: Sequence[int], n_max: int, tau_pad: float = 0.2, eager_max_buc
 # --------------------------------------------------------------------------
 # Sec. 3.5: compaction layout
 # --------------------------------------------------------------------------
-def segment_layout(ctx_len, L_star, n_max: int, tau_pad: float = 0.2, eager_max_bucket: int = 4):
+def segment_layout(ctx_len, L_star, n_max: int, tau_pad: float = 0.2, eager_max_bucket: int = 4, bucket_min: int = 8):
     """Rows kept per sequence after truncation and routing (Sec. 3.4-3.5).
 
     A static-graph group pads each response to the group's bucket (those rows
@@ -190,7 +191,7 @@ def segment_layout(ctx_len, L_star, n_max: int, tau_pad: float = 0.2, eager_max_
     ctx_len = np.asarray(ctx_len, dtype=np.int64)
     L_star = np.asarray(L_star, dtype=np.int64)
     seg = ctx_len + L_star
-    for g in route(L_star, n_max, tau_pad, eager_max_bucket):
+    for g in route(L_star, n_max, tau_pad, eager_max_bucket, bucket_min):
         if g["path"] == PATH_STATIC:
             for i in g["members"]:
                 seg[i] = ctx_len[i] + g["bucket"]

@@ -17,7 +17,7 @@ def _cases(name):
 
 @pytest.mark.parametrize("case", _cases("routing_cases.json"), ids=lambda c: c["name"])
 def test_route_golden(case):
-    got = oracle.route(case["L_star"], case["N"], case["tau_pad"])
+    got = oracle.route(case["L_star"], case["N"], case["tau_pad"], bucket_min=case.get("bucket_min", 8))
     assert len(got) == len(case["groups"])
     for g, e in zip(got, case["groups"]):
         assert g["bucket"] == e["bucket"] and g["members"] == e["members"] and g["path"] == e["path"]
@@ -28,6 +28,9 @@ def test_bucket_set_shape():
     assert oracle.bucket_set(1024) == [8, 16, 32, 64, 128, 256, 512, 1024]
     assert oracle.bucket_set(100) == [8, 16, 32, 64, 100]
     assert oracle.bucket_set(8) == [8]
+    assert oracle.bucket_set(1024, 64) == [64, 128, 256, 512, 1024]
+    assert oracle.bucket_set(50, 64) == [50]
+    assert oracle.bucket_set(100, 1) == [1, 2, 4, 8, 16, 32, 64, 100]
     for N in (100, 512, 2048):
         for L in range(1, N + 1, 7):
             b = oracle.bucket_of(L, N)
