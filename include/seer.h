@@ -78,6 +78,7 @@ typedef struct {
   int window;            /* look-ahead window size w [3] */
   double tau_pad;        /* padding waste threshold for the static path [0.2] */
   int eager_max_bucket;  /* buckets <= this go to the eager path [4] */
+  int bucket_min;        /* smallest micro-bucket; the set doubles from it up to N [8] */
 } seer_params;
 
 /* Device pointers of one block's weights: f16 for a bf16 or f16 layer (make
@@ -157,8 +158,8 @@ seer_status seer_snr_scan(const int32_t* counts, int B, int N, int F, const seer
 /* ---------------------------------------------------------------------------
  * Routing + device-resident compaction (Sec. 3.4-3.5), one fused kernel.
  *
- * Groups the sequences by micro-bucket (smallest of {8,16,...,<N} U {N} that
- * holds L*_b), computes each group's padding waste ratio (Eq. 4) and path:
+ * Groups the sequences by micro-bucket (smallest of {m, 2m, 4m, ..., <N} U {N}
+ * that holds L*_b, m = params->bucket_min, 8 in the paper), computes each group's padding waste ratio (Eq. 4) and path:
  * eager if bucket <= eager_max_bucket or the group has one member, else
  * static if rho <= tau_pad, else varlen.  Static members keep ctx_b + bucket
  * rows (the rows past ctx_b + L*_b are padding, masked as keys), the others

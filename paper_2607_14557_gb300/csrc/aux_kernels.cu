@@ -272,7 +272,7 @@ __global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restri
                                                          const int* __restrict__ cu_full,
                                                          const int* __restrict__ ctx_len,
                                                          const int* __restrict__ L_star, int B, int N, int T_cap,
-                                                         double tau_pad, int eager_max_bucket,
+                                                         double tau_pad, int eager_max_bucket, int bucket_min,
                                                          uint8_t* __restrict__ x_packed, int* cu_out, int* kv_out,
                                                          int* meta_out, int* host_ctrl, int epoch, int* err) {
   extern __shared__ int dyn[];
@@ -283,7 +283,7 @@ __global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restri
 
   if (threadIdx.x == 0) {
     int nb = 0;
-    for (int b = 8; b < N && nb < kCtrlMaxGroups - 1; b *= 2) rs.bucket[nb++] = b;
+    for (int b = bucket_min; b < N && nb < kCtrlMaxGroups - 1; b *= 2) rs.bucket[nb++] = b;
     rs.bucket[nb++] = N;
     rs.n_buckets = nb;
     for (int k = 0; k < nb; ++k) { rs.count[k] = 0; rs.sum[k] = 0; }
@@ -480,8 +480,8 @@ cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_j
 
 cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_full, const int* ctx_len,
                               const int* L_star, int B, int d, int N, int T_cap, double tau_pad,
-                              int eager_max_bucket, void* x_packed, int* cu_out, int* kv_out, int* meta_out,
-                              int* host_ctrl_dev, int epoch, int* err, int num_sms, cudaStream_t st) {
+                              int eager_max_bucket, int bucket_min, void* x_packed, int* cu_out, int* kv_out,
+                              int* meta_out, int* host_ctrl_dev, int epoch, int* err, int num_sms, cudaStream_t st) {
   const size_t sm = static_cast<size_t>(3 * B + 1) * sizeof(int);
   if (sm > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(pack_route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -493,7 +493,7 @@ cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   pack_route_kernel<<<blocks, 256, sm, st>>>(reinterpret_cast<const uint8_t*>(x_full), d * elem_bytes, cu_full,
-                                             ctx_len, L_star, B, N, T_cap, tau_pad, eager_max_bucket,
+                                             ctx_len, L_star, B, N, T_cap, tau_pad, eager_max_bucket, bucket_min,
                                              reinterpret_cast<uint8_t*>(x_packed), cu_out, kv_out, meta_out,
                                              host_ctrl_dev, epoch, err);
   return cudaGetLastError();

@@ -101,7 +101,8 @@ cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_j
                             int* L_star, int* i_star, cudaStream_t st);
 cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_full, const int* ctx_len,
                               const int* L_star, int B, int d, int N, int T_cap, double tau_pad,
-                              int eager_max_bucket, void* x_packed, int* cu_out, int* kv_out, int* meta_out,
+                              int eager_max_bucket, int bucket_min, void* x_packed, int* cu_out, int* kv_out,
+                              int* meta_out,
                               int* host_ctrl_dev, int epoch, int* err, int num_sms, cudaStream_t st);
 
 // Sets the message returned by seer_last_error() on this thread.

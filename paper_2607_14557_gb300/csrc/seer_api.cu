@@ -604,6 +604,7 @@ seer_status seer_pack_ragged(const void* x_full, seer_dtype dt, const int32_t* c
   if (!x_full || !cu_full || !ctx_len || !L_star || !x_packed || !cu_out || !kv_len_out || !meta_out)
     return fail(SEER_ERR_INVALID_ARG, "pack: null pointer");
   if (B <= 0 || d <= 0 || N <= 0 || T_capacity < 0) return fail(SEER_ERR_INVALID_ARG, "pack: bad sizes");
+  if (params->bucket_min < 1) return fail(SEER_ERR_INVALID_ARG, "pack: bucket_min must be >= 1");
   const int es = static_cast<int>(esize(dt));
   if ((static_cast<long>(d) * es) % 16 != 0) return fail(SEER_ERR_UNSUPPORTED, "pack: rows must be a multiple of 16 bytes");
   if (!aligned16(x_full) || !aligned16(x_packed)) return fail(SEER_ERR_UNSUPPORTED, "pack: 16-byte aligned pointers required");
@@ -620,7 +621,8 @@ seer_status seer_pack_ragged(const void* x_full, seer_dtype dt, const int32_t* c
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   Phase ph(PH_PACK, st);
   SEER_CUDA(launch_pack_route(x_full, es, cu_full, ctx_len, L_star, B, d, N, T_capacity, params->tau_pad,
-                              params->eager_max_bucket, x_packed, cu_out, kv_len_out, meta_out, hc_dev, epoch, di->err,
+                              params->eager_max_bucket, params->bucket_min, x_packed, cu_out, kv_len_out, meta_out,
+                              hc_dev, epoch, di->err,
                               di->num_sms, st),
             "pack launch");
   return SEER_OK;

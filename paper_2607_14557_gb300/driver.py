@@ -230,7 +230,7 @@ class SeerPath:
         kv_all = torch.empty(B, **i32)
         meta = torch.empty(S.CTRL_WORDS, **i32)
         p = self.params
-        no_static = S.make_params(p.act_eps, p.tau_jump, p.gamma, p.window, -1.0, p.eager_max_bucket)
+        no_static = S.make_params(p.act_eps, p.tau_jump, p.gamma, p.window, -1.0, p.eager_max_bucket, p.bucket_min)
         S.seer_pack_ragged(x_full, self.dtype, cu_full, ctx_len, L_pad, B, self.dims.d_model, self.N, T, no_static, x,
                            cu, kv_all, meta, None, 0, stream=stream)
         kv = torch.as_tensor((ctx + L).astype(np.int32)).to(dev)

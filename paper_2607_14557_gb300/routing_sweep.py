@@ -3,6 +3,7 @@ Eqs. 3-4) as the padding-waste threshold tau_pad and the batch size vary, next
 to the naive batch-max padding and the untruncated window.
 
     python -m paper_2607_14557_gb300.routing_sweep [--batches 16,32,64,128] [--taus 0.1,0.2,...,0.9]
+                                                   [--bucket-mins 8,16,32,64]
 
 Lengths follow the ragged 8B-layer workload (visual 729k tokens with k in
 1..5, prompt 32..128, window 1024, planted boundary b in 16..400; L* = b + 1);
@@ -10,7 +11,8 @@ hidden states and weights are random device tensors (the timing does not
 depend on their values, and detection is not part of this sweep).  For every
 (batch, tau_pad) the route is built by the library's pack kernel and the
 layer is timed with CUDA events over `--reps` calls; one JSON line per point.
-tau_pad < 0 gives the all-varlen layout (no bucket padding).
+tau_pad < 0 gives the all-varlen layout (no bucket padding).  --bucket-mins sets the
+smallest micro-bucket of the doubling bucket set (the paper's set starts at 8).
 """
 from __future__ import annotations
 
@@ -54,7 +56,7 @@ def _time(fn, reps):
     return a.elapsed_time(b) / reps
 
 
-def sweep(batch, taus, reps, d=4096, H=32, F=12288, N=1024, seed=0):
+def sweep(batch, taus, reps, d=4096, H=32, F=12288, N=1024, seed=0, bucket_min=8):
     dev = torch.device("cuda", 0)
     ctx, L = _lengths(batch, seed)
     full = ctx + N
@@ -70,7 +72,7 @@ def sweep(batch, taus, reps, d=4096, H=32, F=12288, N=1024, seed=0):
     out = []
 
     def point(tau):
-        path = D.SeerPath(dims, "bf16", batch, N, T_full, S.make_params(0.0, tau_pad=tau), dev)
+        path = D.SeerPath(dims, "bf16", batch, N, T_full, S.make_params(0.0, tau_pad=tau, bucket_min=bucket_min), dev)
         path.L_star.copy_(L_d)
         path.pack(x_full, cu_d, ctx_d)
         route = path.route()
@@ -84,7 +86,7 @@ def sweep(batch, taus, reps, d=4096, H=32, F=12288, N=1024, seed=0):
     for tau in taus:
         path, route, seg, kv, ms = point(tau)
         paths = [grp["path"] for grp in route["groups"]]
-        out.append({"batch": batch, "tau_pad": tau, "ms": ms, "tokens_executed": int(seg.sum()),
+        out.append({"batch": batch, "tau_pad": tau, "bucket_min": bucket_min, "ms": ms, "tokens_executed": int(seg.sum()),
                     "pad_rows": route["pad_rows"], "groups": len(route["groups"]),
                     "static_groups": paths.count(0), "varlen_groups": paths.count(1), "eager_groups": paths.count(2),
                     "flops_executed_over_valid": flops(seg, kv) / valid})
@@ -109,10 +111,12 @@ def main(argv=None):
     ap.add_argument("--batches", default="16,32,64,128")
     ap.add_argument("--taus", default="-1,0.1,0.2,0.3,0.4,0.5,0.6,0.7,0.8,0.9")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--bucket-mins", default="8")
     args = ap.parse_args(argv)
-    for b in [int(v) for v in args.batches.split(",")]:
-        for line in sweep(b, [float(t) for t in args.taus.split(",")], args.reps):
-            print(json.dumps(line), flush=True)
+    for bm in [int(v) for v in args.bucket_mins.split(",")]:
+        for b in [int(v) for v in args.batches.split(",")]:
+            for line in sweep(b, [float(t) for t in args.taus.split(",")], args.reps, bucket_min=bm):
+                print(json.dumps(line), flush=True)
         assert S.seer_check_device() == 0
         torch.cuda.empty_cache()
 

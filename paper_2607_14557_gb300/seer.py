@@ -43,7 +43,8 @@ class seer_dims(ctypes.Structure):
 
 class seer_params(ctypes.Structure):
     _fields_ = [("act_eps", ctypes.c_float), ("tau_jump", ctypes.c_double), ("gamma", ctypes.c_double),
-                ("window", ctypes.c_int), ("tau_pad", ctypes.c_double), ("eager_max_bucket", ctypes.c_int)]
+                ("window", ctypes.c_int), ("tau_pad", ctypes.c_double), ("eager_max_bucket", ctypes.c_int),
+                ("bucket_min", ctypes.c_int)]
 
 
 class seer_layer_weights(ctypes.Structure):
@@ -142,8 +143,9 @@ def make_dims(d_model, n_heads, head_dim, d_ff, rms_eps=1e-5, rope_theta=0.0) ->
     return seer_dims(d_model, n_heads, head_dim, d_ff, rms_eps, rope_theta)
 
 
-def make_params(act_eps, tau_jump=0.03, gamma=0.6, window=3, tau_pad=0.2, eager_max_bucket=4) -> seer_params:
-    return seer_params(act_eps, tau_jump, gamma, window, tau_pad, eager_max_bucket)
+def make_params(act_eps, tau_jump=0.03, gamma=0.6, window=3, tau_pad=0.2, eager_max_bucket=4,
+                bucket_min=8) -> seer_params:
+    return seer_params(act_eps, tau_jump, gamma, window, tau_pad, eager_max_bucket, bucket_min)
 
 
 def make_weights(w_qkv, w_o, w_gate, w_up, w_down, g_attn, g_mlp) -> seer_layer_weights:

@@ -282,13 +282,13 @@ def test_detect_boundary_planted(dtype, seed):
 
 
 # ------------------------------------------------------------------ routing + pack (S3 + S4)
-def _pack_case(dtype, ctx, L_star, N, d, tau_pad=0.2, seed=0, extra_cap=50):
+def _pack_case(dtype, ctx, L_star, N, d, tau_pad=0.2, seed=0, extra_cap=50, bucket_min=8):
     rng = _rng(seed)
     B = len(ctx)
     full = np.asarray(ctx) + N
     cu_full = np.concatenate([[0], np.cumsum(full)])
     x = synth.round_storage(rng.standard_normal((int(cu_full[-1]), d)), dtype)
-    seg, kv, cu = oracle.segment_layout(ctx, L_star, N, tau_pad)
+    seg, kv, cu = oracle.segment_layout(ctx, L_star, N, tau_pad, bucket_min=bucket_min)
     ref_rows = oracle.pack_rows(x, cu_full, seg)
     T_cap = int(cu[-1]) + extra_cap
     out = torch.full((T_cap, d), 5.0, dtype=tdtype(dtype), device=cuda())
@@ -296,7 +296,7 @@ def _pack_case(dtype, ctx, L_star, N, d, tau_pad=0.2, seed=0, extra_cap=50):
     kv_out = torch.empty(B, dtype=torch.int32, device=cuda())
     meta = torch.empty(S.CTRL_WORDS, dtype=torch.int32, device=cuda())
     hctrl = torch.zeros(S.CTRL_WORDS, dtype=torch.int32).pin_memory()
-    p = S.make_params(0.0, tau_pad=tau_pad)
+    p = S.make_params(0.0, tau_pad=tau_pad, bucket_min=bucket_min)
     S.seer_pack_ragged(to_dev(x, dtype), dtype, i32(cu_full), i32(ctx), i32(L_star), B, d, N, T_cap, p, out, cu_out,
                        kv_out, meta, hctrl, 9)
     ctrl = torch.zeros(S.CTRL_WORDS, dtype=torch.int32)
@@ -310,7 +310,7 @@ def _pack_case(dtype, ctx, L_star, N, d, tau_pad=0.2, seed=0, extra_cap=50):
     m = meta.cpu().numpy()
     c = ctrl.numpy()
     np.testing.assert_array_equal(m, c)
-    groups = oracle.route(L_star, N, tau_pad)
+    groups = oracle.route(L_star, N, tau_pad, bucket_min=bucket_min)
     assert c[0] == 9 and c[1] == cu[-1] and c[2] == seg.max() and c[4] == len(groups)
     assert c[5] == sum(1 << p_ for p_ in {g["path"] for g in groups})
     pad_ref = sum(g["bucket"] * len(g["members"]) - sum(L_star[i] for i in g["members"])
@@ -340,3 +340,11 @@ def test_pack_route_untruncated_is_identity_layout():
     ctx = [40, 41, 42]
     N = 96
     _pack_case("bf16", ctx, [N, N, N], N, 256, seed=3)
+
+
+@pytest.mark.parametrize("bucket_min", [1, 16, 64, 1024])
+def test_pack_route_bucket_set_variants(bucket_min):
+    # the smallest micro-bucket moves the group boundaries (routing ablation)
+    ctx = [100, 50, 70, 30, 10, 64, 64, 20]
+    L = [120, 128, 110, 125, 300, 5, 16, 3]
+    _pack_case("bf16", ctx, L, 1024, 256, seed=30 + bucket_min, bucket_min=bucket_min)
