@@ -336,6 +336,14 @@ const char* seer_last_error(void);
  * out, 4 boundary out of range, 5 capacity exceeded). */
 seer_status seer_check_device(int* code_out);
 
+/* Failure-detection self-test: enqueues a kernel whose pipeline wait can
+ * never complete (an mbarrier that no thread arrives on).  Like every wait
+ * in the library's kernels it gives up after a time limit, here limit_us
+ * (1 .. 1e7), records the timeout code (3) in the device error word and
+ * returns, so the context stays usable; seer_check_device then reports
+ * SEER_ERR_DEVICE with code 3.  Enqueues only; never waits. */
+seer_status seer_selftest_wait_timeout(int limit_us, void* stream);
+
 /* Per-phase timing with CUDA events recorded on the call's stream.
  * Phases: 0 detect GEMM, 1 SNR scan, 2 pack, 3 norm1, 4 QKV, 5 attention,
  * 6 O proj, 7 norm2, 8 gate/up, 9 down, 10 K/V cache copies and prefix

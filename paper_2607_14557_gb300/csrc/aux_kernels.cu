@@ -201,6 +201,20 @@ __global__ void resp_layout_kernel(const int* cu, const int* ctx, int B, int* cu
   }
 }
 
+// ------------------------------------------------------------------ wait self-test
+// A pipeline wait that can never complete (an mbarrier nothing arrives on),
+// bounded by limit_ns: the same give-up path every tcgen05 kernel's waits
+// take, recording kErrTimeout instead of hanging.
+__global__ void wait_selftest_kernel(uint64_t limit_ns, int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  abort_flag = 0;
+  fence_barrier_init();
+  mbar_wait_for(&bar, 0, &abort_flag, err, limit_ns);
+}
+
 // ------------------------------------------------------------------ SNR scan
 // Sec. 3.3: first 0-based i in [1, N-w] with
 //   jump  = min(s_i .. s_{i+w-1}) - s_{i-1} >= tau_jump
@@ -468,6 +482,11 @@ cudaError_t launch_rows_copy(const void* src, long src_ld, int src_c0, void* dst
 cudaError_t launch_resp_layout(const int* cu, const int* ctx, int B, int* cu_resp, int* cu_ctx, int* err,
                                cudaStream_t st) {
   resp_layout_kernel<<<1, 32, 0, st>>>(cu, ctx, B, cu_resp, cu_ctx, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(uint64_t limit_ns, int* err, cudaStream_t st) {
+  wait_selftest_kernel<<<1, 32, 0, st>>>(limit_ns, err);
   return cudaGetLastError();
 }
 

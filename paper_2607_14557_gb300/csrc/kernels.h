@@ -96,6 +96,8 @@ cudaError_t launch_rows_copy(const void* src, long src_ld, int src_c0, void* dst
 // cu_ctx = exclusive sums of ctx; cu_resp[b] = cu[b] - cu_ctx[b] (either output may be null).
 cudaError_t launch_resp_layout(const int* cu, const int* ctx, int B, int* cu_resp, int* cu_ctx, int* err,
                                cudaStream_t st);
+// A bounded wait on a barrier that never completes (records kErrTimeout).
+cudaError_t launch_wait_selftest(uint64_t limit_ns, int* err, cudaStream_t st);
 cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, cudaStream_t st);
 cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,
                             int* L_star, int* i_star, cudaStream_t st);

@@ -460,6 +460,15 @@ seer_status seer_check_device(int* code_out) {
   return SEER_OK;
 }
 
+seer_status seer_selftest_wait_timeout(int limit_us, void* stream) {
+  if (limit_us < 1 || limit_us > 10000000) return fail(SEER_ERR_INVALID_ARG, "selftest: limit_us must be in [1, 1e7]");
+  DeviceInfo* di;
+  SEER_TRY(device_info(&di));
+  SEER_CUDA(launch_wait_selftest(static_cast<uint64_t>(limit_us) * 1000ull, di->err, static_cast<cudaStream_t>(stream)),
+            "wait selftest launch");
+  return SEER_OK;
+}
+
 seer_status seer_profile_enable(int on) {
   std::lock_guard<std::mutex> lk(g_prof.mu);
   g_prof.on = on != 0;

@@ -90,6 +90,7 @@ def lib() -> ctypes.CDLL:
             "seer_attention": [vp, vp, i32, vp, vp, i32, i32, i32, i32, vp, sz, vp],
             "seer_attention_noalloc": [vp, vp, i32, vp, vp, i32, i32, i32, i32, vp],
             "seer_check_device": [ctypes.POINTER(ctypes.c_int)],
+            "seer_selftest_wait_timeout": [i32, vp],
             "seer_profile_enable": [i32],
             "seer_profile_reset": [],
             "seer_profile_read": [vp, vp],
@@ -276,3 +277,7 @@ def seer_num_sms() -> int:
 
 def seer_version() -> str:
     return lib().seer_version().decode()
+
+
+def seer_selftest_wait_timeout(limit_us: int, stream=None):
+    _check(lib().seer_selftest_wait_timeout(limit_us, _stream(stream)))
