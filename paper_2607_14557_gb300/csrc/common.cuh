@@ -291,6 +291,22 @@ enum ElemType : int { kF32 = 0, kBF16 = 1, kF16 = 2 };
 
 __device__ __forceinline__ int elect_lane0() { return (threadIdx.x & 31) == 0; }
 
+// Raises a kernel's dynamic shared-memory limit once per device (the setting
+// belongs to the current device's context, so every device needs its own).
+template <typename Kernel>
+inline cudaError_t set_smem_limit_once(Kernel kernel, int bytes, bool (&done)[64]) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!done[dev]) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  return cudaSuccess;
+}
+
 // ---------------------------------------------------------------- rotary embedding
 // Inverse frequency theta^(-2i/dh) of pair i, computed in double and split into
 // a float head and tail (hi + lo equals it to ~2^-48 relative).

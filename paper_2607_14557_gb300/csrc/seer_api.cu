@@ -88,13 +88,13 @@ bool is16(seer_dtype dt) { return dt == SEER_BF16 || dt == SEER_F16; }
 size_t esize(seer_dtype dt) { return dt == SEER_F32 ? 4 : 2; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-
 // ------------------------------------------------------------ TMA descriptors
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 
-// Row-major [rows, cols] 16-bit matrix with leading dimension ld elements,
-// boxes of 64 columns (128 bytes, 128-byte swizzle) x box_rows rows.
+// Row-major [rows, cols] 16-bit matrix with leading dimension ld elements, in
+// boxes of box_cols columns x box_rows rows: 128-byte swizzle for operand
+// tiles (64 columns = 128 bytes), none for the GEMM epilogue's store chunks.
 seer_status make_map16(CUtensorMap* m, const void* base, seer_dtype dt, uint64_t rows, uint64_t cols, uint64_t ld,
                        uint32_t box_rows, uint32_t box_cols = 64, bool swizzle128 = true) {
   std::call_once(g_encode_once, [] {

@@ -448,12 +448,9 @@ __global__ void attn_schedule_kernel(const int* cu, const int* cu_kv, const int*
 
 template <bool F16>
 cudaError_t launch_typed(const CUtensorMap& mQ, const CUtensorMap& mKV, const AttnParams& p, int grid, cudaStream_t st) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc_attn_kernel<F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static bool attr_set[64] = {};
+  cudaError_t e = set_smem_limit_once(tc_attn_kernel<F16>, SMEM_BYTES, attr_set);
+  if (e != cudaSuccess) return e;
   if (grid <= 0) return cudaSuccess;
   tc_attn_kernel<F16><<<grid, THREADS, SMEM_BYTES, st>>>(mQ, mKV, p);
   return cudaGetLastError();

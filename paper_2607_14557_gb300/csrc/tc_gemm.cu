@@ -402,12 +402,9 @@ __global__ void __launch_bounds__(THREADS, 1)
 template <int MODE>
 cudaError_t launch_mode(const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1, const CUtensorMap& mC,
                         const GemmParams& p, int num_sms, cudaStream_t st) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static bool attr_set[64] = {};
+  cudaError_t e = set_smem_limit_once(tc_gemm_kernel<MODE>, SMEM_BYTES, attr_set);
+  if (e != cudaSuccess) return e;
   long num_m;
   if (MODE == kGemmCount) num_m = static_cast<long>(p.B) * ((p.Nw + BM - 1) / BM);
   else num_m = (p.M_cap + BM - 1) / BM;
