@@ -2,11 +2,16 @@
 
     python -m paper_2607_14557_gb300.kernel_bench attention --lens 3100x8 [--heads 32] [--dtype f16]
     python -m paper_2607_14557_gb300.kernel_bench linear --M 35194 --N 12288 --K 4096 [--dtype f16]
+    python -m paper_2607_14557_gb300.kernel_bench pack [--batch 16 --window 1024 --d 4096]
+    python -m paper_2607_14557_gb300.kernel_bench scan [--batch 16 --window 1024]
 
 Each call runs the kernel `--warmup` times, then times `--reps` calls with CUDA
 events on the launching stream and prints one JSON line (ms per call and
 TFLOP/s of the algorithmic work: 4*d*sum(L^2) for attention, 2*M*N*K for a
-linear).  Inputs are random and resident in device memory; no output is checked
+linear; GB/s of algorithmic bytes for pack (each kept row read and written
+once) and scan (each count read once)).  pack and scan use the lengths of the
+ragged 8B-layer workload (visual 729k, k in 1..5; prompt 32..128; boundary
+16..400).  Inputs are random and resident in device memory; no output is checked
 (the parity tests do that).  Used for per-kernel timings and small ncu captures.
 """
 from __future__ import annotations
@@ -79,6 +84,48 @@ def linear(args) -> dict:
             "tflops": 2.0 * args.M * args.N * args.K / (ms * 1e-3) / 1e12}
 
 
+def _ragged_lengths(batch, seed):
+    rng = np.random.default_rng(seed)
+    ctx = 729 * rng.integers(1, 6, batch) + rng.integers(32, 129, batch)
+    return ctx, rng.integers(16, 401, batch) + 1
+
+
+def pack(args) -> dict:
+    dev = torch.device("cuda", 0)
+    B, N, d = args.batch, args.window, args.d
+    ctx, L = _ragged_lengths(B, args.seed)
+    cu_full = np.concatenate([[0], np.cumsum(ctx + N)]).astype(np.int32)
+    T = int(cu_full[-1])
+    g = torch.Generator(device=dev).manual_seed(args.seed)
+    x = torch.randn((T, d), device=dev, generator=g).to(torch.bfloat16)
+    out = torch.empty_like(x)
+    i32 = lambda a: torch.as_tensor(np.asarray(a, dtype=np.int32)).to(dev)
+    cu_d, ctx_d, L_d = i32(cu_full), i32(ctx), i32(L)
+    cu, kv = torch.empty(B + 1, dtype=torch.int32, device=dev), torch.empty(B, dtype=torch.int32, device=dev)
+    meta = torch.empty(S.CTRL_WORDS, dtype=torch.int32, device=dev)
+    p = S.make_params(0.0)
+    ms = _time(lambda: S.seer_pack_ragged(x, "bf16", cu_d, ctx_d, L_d, B, d, N, T, p, out, cu, kv, meta),
+               args.warmup, args.reps)
+    rows = int(cu[-1].item())
+    return {"kernel": "pack", "batch": B, "window": N, "d": d, "rows_kept": rows, "rows_full": T, "ms": ms,
+            "gbs": 2.0 * rows * d * 2 / (ms * 1e-3) / 1e9}
+
+
+def scan(args) -> dict:
+    dev = torch.device("cuda", 0)
+    B, N, F = args.batch, args.window, 12288
+    _, L = _ragged_lengths(B, args.seed)
+    rng = np.random.default_rng(args.seed)
+    counts = rng.integers(100, 400, (B, N))
+    for b in range(B):
+        counts[b, int(L[b]) - 1:] += 6000                # planted plateau past the boundary
+    c = torch.as_tensor(counts.astype(np.int32).ravel()).to(dev)
+    Ls, Is = torch.empty(B, dtype=torch.int32, device=dev), torch.empty(B, dtype=torch.int32, device=dev)
+    p = S.make_params(0.0)
+    ms = _time(lambda: S.seer_snr_scan(c, B, N, F, p, Ls, Is), args.warmup, args.reps)
+    return {"kernel": "scan", "batch": B, "window": N, "ms": ms, "gbs": B * N * 4 / (ms * 1e-3) / 1e9}
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     sub = ap.add_subparsers(dest="kernel", required=True)
@@ -94,8 +141,19 @@ def main(argv=None):
         p.add_argument("--warmup", type=int, default=3)
         p.add_argument("--reps", type=int, default=10)
         p.add_argument("--seed", type=int, default=0)
+    pp = sub.add_parser("pack")
+    pp.add_argument("--batch", type=int, default=16)
+    pp.add_argument("--window", type=int, default=1024)
+    pp.add_argument("--d", type=int, default=4096)
+    ps = sub.add_parser("scan")
+    ps.add_argument("--batch", type=int, default=16)
+    ps.add_argument("--window", type=int, default=1024)
+    for q in (pp, ps):
+        q.add_argument("--warmup", type=int, default=3)
+        q.add_argument("--reps", type=int, default=10)
+        q.add_argument("--seed", type=int, default=0)
     args = ap.parse_args(argv)
-    res = attention(args) if args.kernel == "attention" else linear(args)
+    res = {"attention": attention, "linear": linear, "pack": pack, "scan": scan}[args.kernel](args)
     assert S.seer_check_device() == 0, "a kernel recorded a device-side error"
     print(json.dumps(res), flush=True)
 
