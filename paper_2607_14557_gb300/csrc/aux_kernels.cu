@@ -216,6 +216,7 @@ __global__ void wait_selftest_kernel(uint64_t limit_ns, int* err) {
 }
 
 // ------------------------------------------------------------------ SNR scan
+constexpr int kScanSmemInts = 12288;   // 48 KB of staged counts per sequence at most
 // Sec. 3.3: first 0-based i in [1, N-w] with
 //   jump  = min(s_i .. s_{i+w-1}) - s_{i-1} >= tau_jump
 //   noise = max(s_i .. s_{i+w-1}) - min(..)  <= gamma * jump,   s = c / F,
@@ -227,6 +228,14 @@ __global__ void __launch_bounds__(32) snr_scan_kernel(const int* __restrict__ co
   const int b = blockIdx.x;
   const int lane = threadIdx.x;
   const int* c = counts + static_cast<size_t>(b) * N;
+  // the sequence's counts staged in shared memory by one coalesced pass (all
+  // loads in flight at once) when they fit; the scan then reads them there
+  extern __shared__ int staged[];
+  if (N <= kScanSmemInts) {
+    for (int i = lane; i < N; i += 32) staged[i] = c[i];
+    __syncwarp();
+    c = staged;
+  }
   const double Fd = static_cast<double>(F);
   int found = -1;
   const int last = N - window;   // inclusive
@@ -399,7 +408,8 @@ __global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restri
     }
   }
 
-  // ---- copy rows, one warp per row, 16-byte vectors
+  // ---- copy rows, one warp per row, 16-byte vectors; four loads in flight
+  // per lane before their stores
   const int total = min(rs.total, T_cap);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int vec = row_bytes / 16;
@@ -412,7 +422,15 @@ __global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restri
     const int src = cu_full[lo] + (r - cus[lo]);
     const uint4* s = reinterpret_cast<const uint4*>(x_full + static_cast<size_t>(src) * row_bytes);
     uint4* dst = reinterpret_cast<uint4*>(x_packed + static_cast<size_t>(r) * row_bytes);
-    for (int v = lane; v < vec; v += 32) dst[v] = s[v];
+    int v = lane;
+    for (; v + 96 < vec; v += 128) {
+      const uint4 a0 = s[v], a1 = s[v + 32], a2 = s[v + 64], a3 = s[v + 96];
+      dst[v] = a0;
+      dst[v + 32] = a1;
+      dst[v + 64] = a2;
+      dst[v + 96] = a3;
+    }
+    for (; v < vec; v += 32) dst[v] = s[v];
   }
 }
 
@@ -493,7 +511,8 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, int* err, cudaStream_t st) {
 cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,
                             int* L_star, int* i_star, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
-  snr_scan_kernel<<<B, 32, 0, st>>>(counts, N, F, tau_jump, gamma, window, L_star, i_star);
+  const size_t sm = N <= kScanSmemInts ? static_cast<size_t>(N) * sizeof(int) : 0;
+  snr_scan_kernel<<<B, 32, sm, st>>>(counts, N, F, tau_jump, gamma, window, L_star, i_star);
   return cudaGetLastError();
 }
 
