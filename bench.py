@@ -332,6 +332,10 @@ def run_stack(args, wl, world, rank, local):
             "speedup_vs_truncated_uncached": ms_seer / ms_cached_total,
             "tokens_per_s": (T_full + (n_steps - 1) * T_valid) * nl / (ms_cached_total * 1e-3),
             "clocks": clk_c.summary()},
+        "roofline": {"kernel": "the truncated layer's kernels under graph replay (steps 1..%d)" % (n_steps - 1),
+                     "bound": "tensor", "achieved": tflops_rest, "peak": pk["bf16_tflops_sustained"],
+                     "unit": "TFLOP/s", "frac": tflops_rest / pk["bf16_tflops_sustained"], "traffic": None,
+                     "peak_source": f"{src} bf16 dense, sustained (a {ms_rest / 1e3:.0f} s region under the power cap)"},
         "gpu_launches": nl * 8 * (2 * n_steps) + 3 + (nl * 8 + 4)
                         + (nl * 8 + 3) + nl * 13 + (n_steps - 2) * (2 + nl * 9), "clocks": clk.summary(),
         "peak_source": src,
@@ -508,12 +512,15 @@ def main():
             kernels[name]["gbs"] = by / (kernels[name]["ms_per_launch"] * 1e-3) / 1e9
     gu = kernels.get("gate_up", {})
     achieved = gu.get("tflops")
-    peak = pk["bf16_tflops_sustained"]
+    # the timed region is ~0.1 s at full clocks: the burst figure is the denominator
+    # (the sustained one, a seconds-long loop under the power cap, is reported beside it)
+    peak = pk["bf16_tflops"]
     roofline = {"kernel": "tc_gemm_kernel<Swiglu> (gate/up + SwiGLU)", "bound": "tensor", "achieved": achieved,
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak if achieved else None,
+                "frac_of_sustained": achieved / pk["bf16_tflops_sustained"] if achieved else None,
                 "traffic": measured_traffic(wl.index, "gate_up"),
                 "algorithmic_bytes": float(2 * T_exec * d + 2 * 2 * F * d + 2 * T_exec * F),
-                "peak_source": f"{src} bf16 dense, sustained (f16 operands run at the bf16 rate)",
+                "peak_source": f"{src} bf16 dense, burst (f16 operands run at the bf16 rate)",
                 "flops_per_launch": flops_of["gate_up"]}
 
     clocks = clk.summary()
