@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--launch-overlap", default="on", choices=["on", "off"],
+                    help="programmatic dependent launch of the library kernels (default on)")
     return ap.parse_args()
 
 
@@ -312,7 +314,7 @@ def run_stack(args, wl, world, rank, local):
                    "tokens_full": T_full, "tokens_valid": T_valid, "tokens_executed": T_exec, "L_star": L.tolist(),
                    "route": {"groups": r["groups"], "capacity": r["capacity"]},
                    "l2": "inputs larger than L2 (weights %.1f GB)" % (nl * (4 * d * d + 3 * d * F) * 2 / 1e9),
-                   "weights_setup_s": t_weights},
+                   "weights_setup_s": t_weights, "launch_overlap": args.launch_overlap},
         "stack": {"ms_step0_full": ms0, "ms_steps_1_to_%d" % (n_steps - 1): ms_rest, "ms_padded_%d_steps" % n_steps: ms_pad,
                   "speedup_vs_padded": ms_pad / ms_seer,
                   "ideal_ratio": fl_full * n_steps / (fl_full + fl_valid * (n_steps - 1)),
@@ -359,6 +361,9 @@ def main():
     if args.impl == "reference":
         run_reference(args, wl, rank, world)
         return
+    from paper_2607_14557_gb300 import seer as S_
+
+    S_.seer_set_launch_overlap(args.launch_overlap == "on")
     if args.workload == 3:
         run_stack(args, wl, world, rank, local)
         return
@@ -537,7 +542,7 @@ def main():
                    "l2": "inputs larger than L2 (x_full %.0f MB, weights %.0f MB)" % (
                        T_full * d * es / 1e6, (4 * d * d + 3 * d * F) * 2 / 1e6),
                    "route": {"groups": route["groups"], "pad_rows": route["pad_rows"], "capacity": route["capacity"]},
-                   "parallelism": f"replicas x{world}"},
+                   "parallelism": f"replicas x{world}", "launch_overlap": args.launch_overlap},
         "layer": {"ms_truncated": ms_layer, "ms_padded": ms_pad, "tflops": flops_exec / (ms_layer * 1e-3) / 1e12,
                   "frac_of_burst_peak": flops_exec / (ms_layer * 1e-3) / 1e12 / pk["bf16_tflops"],
                   "frac_of_sustained_peak": flops_exec / (ms_layer * 1e-3) / 1e12 / pk["bf16_tflops_sustained"],

@@ -344,6 +344,15 @@ seer_status seer_check_device(int* code_out);
  * SEER_ERR_DEVICE with code 3.  Enqueues only; never waits. */
 seer_status seer_selftest_wait_timeout(int limit_us, void* stream);
 
+/* Launch overlap (programmatic dependent launch).  When on (the default),
+ * each kernel of the library is launched as a programmatic dependent of the
+ * previous kernel in its stream: the GPU may place its blocks while that
+ * kernel finishes, which hides most of the launch gap between consecutive
+ * kernels.  Every kernel waits at entry until the kernels before it have
+ * completed and their writes are visible, so results are the same with the
+ * setting on or off.  Process-wide; returns the previous setting (1 or 0). */
+int seer_set_launch_overlap(int on);
+
 /* Per-phase timing with CUDA events recorded on the call's stream.
  * Phases: 0 detect GEMM, 1 SNR scan, 2 pack, 3 norm1, 4 QKV, 5 attention,
  * 6 O proj, 7 norm2, 8 gate/up, 9 down, 10 K/V cache copies and prefix

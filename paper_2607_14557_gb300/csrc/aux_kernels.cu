@@ -47,6 +47,7 @@ template <int IN, int OUT>
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ x, const void* __restrict__ g,
                                                       void* __restrict__ y, int M_cap, const int* M_dev, int d,
                                                       float eps, int* err) {
+  pdl_enter();
   int M = M_cap;
   if (M_dev != nullptr) {
     const int md = *M_dev;
@@ -86,6 +87,7 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ x
 // Element-wise storage conversion (used once per model for f16 weight copies).
 template <int IN, int OUT>
 __global__ void convert_kernel(const void* __restrict__ src, void* __restrict__ dst, size_t n8) {
+  pdl_enter();
   for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n8;
        i += static_cast<size_t>(gridDim.x) * blockDim.x) {
     float e[8];
@@ -116,6 +118,7 @@ __device__ __forceinline__ void st1(void* base, size_t i, float x) {
 template <int T>
 __global__ void __launch_bounds__(256) rope_kernel(void* __restrict__ qkv, const int* __restrict__ cu, int B, int T_cap,
                                                    int H, int dh, float theta, int* err) {
+  pdl_enter();
   __shared__ float2 tab[64];
   const int half = dh / 2;
   for (int i = threadIdx.x; i < half; i += blockDim.x) tab[i] = rope_inv_freq(i, dh, theta);
@@ -167,6 +170,7 @@ struct RowsCopyArgs {
 };
 
 __global__ void __launch_bounds__(256) rows_copy_kernel(const RowsCopyArgs a) {
+  pdl_enter();
   const int b = blockIdx.y;
   const int s0 = a.src_start[b] + (a.src_add ? a.src_add[b] : 0);
   const int d0 = a.dst_start[b] + (a.dst_add ? a.dst_add[b] : 0);
@@ -188,6 +192,7 @@ __global__ void __launch_bounds__(256) rows_copy_kernel(const RowsCopyArgs a) {
 // cu_ctx = exclusive prefix sums of ctx (B+1 entries); cu_resp[b] = cu[b] -
 // cu_ctx[b]: the offsets of the rows past each segment's first ctx[b] rows.
 __global__ void resp_layout_kernel(const int* cu, const int* ctx, int B, int* cu_resp, int* cu_ctx, int* err) {
+  pdl_enter();
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   int acc = 0;
   for (int b = 0; b <= B; ++b) {
@@ -225,6 +230,7 @@ constexpr int kScanSmemInts = 12288;   // 48 KB of staged counts per sequence at
 __global__ void __launch_bounds__(32) snr_scan_kernel(const int* __restrict__ counts, int N, int F, double tau_jump,
                                                       double gamma, int window, int* __restrict__ L_star,
                                                       int* __restrict__ i_star) {
+  pdl_enter();
   const int b = blockIdx.x;
   const int lane = threadIdx.x;
   const int* c = counts + static_cast<size_t>(b) * N;
@@ -298,6 +304,7 @@ __global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restri
                                                          double tau_pad, int eager_max_bucket, int bucket_min,
                                                          uint8_t* __restrict__ x_packed, int* cu_out, int* kv_out,
                                                          int* meta_out, int* host_ctrl, int epoch, int* err) {
+  pdl_enter();
   extern __shared__ int dyn[];
   int* seg = dyn;              // [B]
   int* cus = dyn + B;          // [B+1]
@@ -442,7 +449,7 @@ cudaError_t launch_rmsnorm(const void* x, int in_type, const void* g, void* y, i
   int blocks = (M_cap + 7) / 8;
   if (blocks > 65535 * 4) blocks = 65535 * 4;
 #define SEER_NORM(I, O) \
-  if (in_type == I && out_type == O) { rmsnorm_kernel<I, O><<<blocks, 256, 0, st>>>(x, g, y, M_cap, M_dev, d, eps, err); return cudaGetLastError(); }
+  if (in_type == I && out_type == O) return launch_kernel(rmsnorm_kernel<I, O>, dim3(blocks), dim3(256), 0, st, x, g, y, M_cap, M_dev, d, eps, err);
   SEER_NORM(kBF16, kF16)
   SEER_NORM(kF16, kF16)
   SEER_NORM(kBF16, kBF16)
@@ -457,7 +464,7 @@ cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type
   const size_t n8 = n / 8;
   const int blocks = static_cast<int>(n8 / 256 + 1 < 4096 ? n8 / 256 + 1 : 4096);
 #define SEER_CONV(I, O) \
-  if (in_type == I && out_type == O) { convert_kernel<I, O><<<blocks, 256, 0, st>>>(src, dst, n8); return cudaGetLastError(); }
+  if (in_type == I && out_type == O) return launch_kernel(convert_kernel<I, O>, dim3(blocks), dim3(256), 0, st, src, dst, n8);
   SEER_CONV(kBF16, kF16)
   SEER_CONV(kF16, kBF16)
   SEER_CONV(kBF16, kF32)
@@ -474,12 +481,11 @@ cudaError_t launch_rope(void* qkv, int type, const int* cu, int B, int T_cap, in
   if (head_dim % 2 != 0 || head_dim > 128) return cudaErrorInvalidValue;
   const int blocks = T_cap < 8 * num_sms ? T_cap : 8 * num_sms;
   switch (type) {
-    case kF32: rope_kernel<kF32><<<blocks, 256, 0, st>>>(qkv, cu, B, T_cap, n_heads, head_dim, theta, err); break;
-    case kF16: rope_kernel<kF16><<<blocks, 256, 0, st>>>(qkv, cu, B, T_cap, n_heads, head_dim, theta, err); break;
-    case kBF16: rope_kernel<kBF16><<<blocks, 256, 0, st>>>(qkv, cu, B, T_cap, n_heads, head_dim, theta, err); break;
+    case kF32: return launch_kernel(rope_kernel<kF32>, dim3(blocks), dim3(256), 0, st, qkv, cu, B, T_cap, n_heads, head_dim, theta, err);
+    case kF16: return launch_kernel(rope_kernel<kF16>, dim3(blocks), dim3(256), 0, st, qkv, cu, B, T_cap, n_heads, head_dim, theta, err);
+    case kBF16: return launch_kernel(rope_kernel<kBF16>, dim3(blocks), dim3(256), 0, st, qkv, cu, B, T_cap, n_heads, head_dim, theta, err);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_rows_copy(const void* src, long src_ld, int src_c0, void* dst, long dst_ld, int dst_c0, int row_bytes,
@@ -493,14 +499,12 @@ cudaError_t launch_rows_copy(const void* src, long src_ld, int src_c0, void* dst
   RowsCopyArgs a{static_cast<const uint8_t*>(src), src_ld, src_c0, static_cast<uint8_t*>(dst), dst_ld, dst_c0, row_bytes,
                  src_start, src_add, len, len_sub, dst_start, dst_add, B, src_rows, dst_rows, err};
   const int gx = (max_rows + 7) / 8 < 64 ? (max_rows + 7) / 8 : 64;
-  rows_copy_kernel<<<dim3(gx, B), 256, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(rows_copy_kernel, dim3(gx, B), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_resp_layout(const int* cu, const int* ctx, int B, int* cu_resp, int* cu_ctx, int* err,
                                cudaStream_t st) {
-  resp_layout_kernel<<<1, 32, 0, st>>>(cu, ctx, B, cu_resp, cu_ctx, err);
-  return cudaGetLastError();
+  return launch_kernel(resp_layout_kernel, dim3(1), dim3(32), 0, st, cu, ctx, B, cu_resp, cu_ctx, err);
 }
 
 cudaError_t launch_wait_selftest(uint64_t limit_ns, int* err, cudaStream_t st) {
@@ -512,8 +516,7 @@ cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_j
                             int* L_star, int* i_star, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
   const size_t sm = N <= kScanSmemInts ? static_cast<size_t>(N) * sizeof(int) : 0;
-  snr_scan_kernel<<<B, 32, sm, st>>>(counts, N, F, tau_jump, gamma, window, L_star, i_star);
-  return cudaGetLastError();
+  return launch_kernel(snr_scan_kernel, dim3(B), dim3(32), sm, st, counts, N, F, tau_jump, gamma, window, L_star, i_star);
 }
 
 cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_full, const int* ctx_len,
@@ -530,11 +533,9 @@ cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_
   const int cap = num_sms * 8;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  pack_route_kernel<<<blocks, 256, sm, st>>>(reinterpret_cast<const uint8_t*>(x_full), d * elem_bytes, cu_full,
-                                             ctx_len, L_star, B, N, T_cap, tau_pad, eager_max_bucket, bucket_min,
-                                             reinterpret_cast<uint8_t*>(x_packed), cu_out, kv_out, meta_out,
-                                             host_ctrl_dev, epoch, err);
-  return cudaGetLastError();
+  return launch_kernel(pack_route_kernel, dim3(blocks), dim3(256), sm, st, reinterpret_cast<const uint8_t*>(x_full),
+                       d * elem_bytes, cu_full, ctx_len, L_star, B, N, T_cap, tau_pad, eager_max_bucket, bucket_min,
+                       reinterpret_cast<uint8_t*>(x_packed), cu_out, kv_out, meta_out, host_ctrl_dev, epoch, err);
 }
 
 }  // namespace seer

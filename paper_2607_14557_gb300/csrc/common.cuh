@@ -10,6 +10,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace seer {
 
 // Device-side error codes (mirrored in include/seer.h, seer_check_device).
@@ -290,6 +292,53 @@ __device__ __forceinline__ void st_global_v8(void* p, uint32_t a0, uint32_t a1, 
 enum ElemType : int { kF32 = 0, kBF16 = 1, kF16 = 2 };
 
 __device__ __forceinline__ int elect_lane0() { return (threadIdx.x & 31) == 0; }
+
+// ---------------------------------------------------------------- programmatic dependent launch
+// Kernels are launched with launch_kernel(), which marks each one as a
+// programmatic dependent of the previous kernel in the stream (when launch
+// overlap is on): the next kernel may be launched, and its blocks placed,
+// before the current one has finished.  Every kernel of the library calls
+// pdl_wait() before anything else: it returns once the kernels it depends on
+// have completed and their writes are visible, so no kernel touches global
+// memory while its predecessor runs.  pdl_trigger() lets the next kernel
+// launch; a kernel calls it only after its own wait, which keeps the chain
+// ordered, and where it calls it sets how long the successor's blocks sit
+// waiting: short kernels trigger at entry, the persistent GEMM once its last
+// MMAs are issued.  Without a predecessor in flight, or when launched
+// normally, the wait returns at once; a kernel that never triggers lets its
+// successor launch when it completes.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_enter() {
+  pdl_wait();
+  pdl_trigger();
+}
+
+bool launch_overlap_enabled();
+
+// Launches `kernel` as a programmatic dependent of the previous kernel in the
+// stream when `overlap` is set, else as an ordinary launch.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_kernel_overlap(bool overlap, void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                         cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = overlap ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                 Args&&... args) {
+  return launch_kernel_overlap(launch_overlap_enabled(), kernel, grid, block, smem, st, std::forward<Args>(args)...);
+}
 
 // Raises a kernel's dynamic shared-memory limit once per device (the setting
 // belongs to the current device's context, so every device needs its own).

@@ -430,10 +430,15 @@ seer_status do_attention(const void* qkv, void* o, seer_dtype dt, const int32_t*
 
 }  // namespace
 
+namespace {
+std::atomic<int> g_launch_overlap{1};
+}  // namespace
+
 namespace seer {
 // Lets other translation units of the library report a message through
 // seer_last_error().
 void set_last_error(const char* msg) { g_msg = msg; }
+bool launch_overlap_enabled() { return g_launch_overlap.load(std::memory_order_relaxed) != 0; }
 }  // namespace seer
 
 extern "C" {
@@ -441,6 +446,8 @@ extern "C" {
 const char* seer_last_error(void) { return g_msg.c_str(); }
 
 const char* seer_version(void) { return "libseer 0.2 (sm_103a)"; }
+
+int seer_set_launch_overlap(int on) { return g_launch_overlap.exchange(on ? 1 : 0); }
 
 int seer_num_sms(void) {
   DeviceInfo* di;

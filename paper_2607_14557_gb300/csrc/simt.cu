@@ -20,6 +20,7 @@ __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)
 template <int MODE>
 __global__ void __launch_bounds__(256) simt_gemm_kernel(const float* __restrict__ A, const float* __restrict__ B0,
                                                         const float* __restrict__ B1, const GemmParams p) {
+  pdl_enter();
   __shared__ float As[TK][TB + 1];
   __shared__ float Bs0[TK][TB + 1];
   __shared__ float Bs1[TK][TB + 1];
@@ -133,6 +134,7 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const float* __restrict_
 // One warp per (query row, head): lanes split the head dimension, keys are
 // visited in order with an online softmax (fp32).
 __global__ void __launch_bounds__(256) simt_attn_kernel(const float* __restrict__ qkv, const AttnParams p) {
+  pdl_enter();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long task = static_cast<long>(blockIdx.x) * 8 + warp;
   const int H = p.n_heads, dh = p.head_dim, D = H * dh;
@@ -208,13 +210,12 @@ cudaError_t launch_simt_gemm(int mode, const float* A, const float* B0, const fl
   if (mtiles > 65535) return cudaErrorInvalidValue;
   dim3 grid(ntiles, mtiles);
   switch (mode) {
-    case kGemmStore: simt_gemm_kernel<kGemmStore><<<grid, 256, 0, st>>>(A, B0, B1, p); break;
-    case kGemmResidual: simt_gemm_kernel<kGemmResidual><<<grid, 256, 0, st>>>(A, B0, B1, p); break;
-    case kGemmSwiglu: simt_gemm_kernel<kGemmSwiglu><<<grid, 256, 0, st>>>(A, B0, B1, p); break;
-    case kGemmCount: simt_gemm_kernel<kGemmCount><<<grid, 256, 0, st>>>(A, B0, B1, p); break;
+    case kGemmStore: return launch_kernel(simt_gemm_kernel<kGemmStore>, grid, dim3(256), 0, st, A, B0, B1, p);
+    case kGemmResidual: return launch_kernel(simt_gemm_kernel<kGemmResidual>, grid, dim3(256), 0, st, A, B0, B1, p);
+    case kGemmSwiglu: return launch_kernel(simt_gemm_kernel<kGemmSwiglu>, grid, dim3(256), 0, st, A, B0, B1, p);
+    case kGemmCount: return launch_kernel(simt_gemm_kernel<kGemmCount>, grid, dim3(256), 0, st, A, B0, B1, p);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_simt_attn(const float* qkv, const AttnParams& p, cudaStream_t st) {
@@ -222,8 +223,7 @@ cudaError_t launch_simt_attn(const float* qkv, const AttnParams& p, cudaStream_t
   if (tasks <= 0) return cudaSuccess;
   const long blocks = (tasks + 7) / 8;
   if (blocks > 0x7fffffffL) return cudaErrorInvalidValue;
-  simt_attn_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(qkv, p);
-  return cudaGetLastError();
+  return launch_kernel(simt_attn_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, qkv, p);
 }
 
 }  // namespace seer

@@ -114,6 +114,7 @@ __device__ __forceinline__ void row_probs(const float* s, float scale_log2, floa
 template <bool F16>
 __global__ void __launch_bounds__(THREADS, 1)
     tc_attn_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mKV, const AttnParams p) {
+  pdl_enter();
   const int u = blockIdx.x;
   if (u >= *p.work_count) return;
   const int4 wk = p.work[u];
@@ -391,6 +392,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 // segments start first.
 __global__ void attn_schedule_kernel(const int* cu, const int* cu_kv, const int* kv_len, int B, int H, int T_cap,
                                      int4* work, int* work_count, int max_units, int* err) {
+  pdl_enter();
   extern __shared__ int sh[];
   int* ntile = sh;           // [B]
   int* kvs = sh + B;         // [B]
@@ -452,8 +454,7 @@ cudaError_t launch_typed(const CUtensorMap& mQ, const CUtensorMap& mKV, const At
   cudaError_t e = set_smem_limit_once(tc_attn_kernel<F16>, SMEM_BYTES, attr_set);
   if (e != cudaSuccess) return e;
   if (grid <= 0) return cudaSuccess;
-  tc_attn_kernel<F16><<<grid, THREADS, SMEM_BYTES, st>>>(mQ, mKV, p);
-  return cudaGetLastError();
+  return launch_kernel(tc_attn_kernel<F16>, dim3(grid), dim3(THREADS), SMEM_BYTES, st, mQ, mKV, p);
 }
 
 }  // namespace
@@ -473,8 +474,8 @@ cudaError_t launch_attn_schedule(const int* cu, const int* cu_kv, const int* kv_
                                          static_cast<int>(sm));
     if (e != cudaSuccess) return e;
   }
-  attn_schedule_kernel<<<1, 256, sm, st>>>(cu, cu_kv, kv_len, B, n_heads, T_cap, work, work_count, max_units, err);
-  return cudaGetLastError();
+  return launch_kernel(attn_schedule_kernel, dim3(1), dim3(256), sm, st, cu, cu_kv, kv_len, B, n_heads, T_cap, work,
+                       work_count, max_units, err);
 }
 
 }  // namespace seer

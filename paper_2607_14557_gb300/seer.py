@@ -103,6 +103,8 @@ def lib() -> ctypes.CDLL:
         L.seer_last_error.argtypes = []
         L.seer_version.restype = ctypes.c_char_p
         L.seer_num_sms.restype = ctypes.c_int
+        L.seer_set_launch_overlap.restype = ctypes.c_int
+        L.seer_set_launch_overlap.argtypes = [ctypes.c_int]
         _lib = L
     return _lib
 
@@ -269,6 +271,12 @@ def seer_profile_read():
     n = (ctypes.c_int32 * N_PHASES)()
     _check(lib().seer_profile_read(ctypes.addressof(ms), ctypes.addressof(n)))
     return {PHASES[i]: (float(ms[i]), int(n[i])) for i in range(N_PHASES)}
+
+
+def seer_set_launch_overlap(on: bool) -> bool:
+    """Turns programmatic dependent launch of the library's kernels on or off
+    (process-wide); returns the previous setting."""
+    return bool(lib().seer_set_launch_overlap(1 if on else 0))
 
 
 def seer_num_sms() -> int:

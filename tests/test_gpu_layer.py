@@ -111,6 +111,25 @@ def test_batch_permutation_is_bit_exact():
         np.testing.assert_array_equal(a, b)
 
 
+def test_launch_overlap_gives_identical_results():
+    # programmatic dependent launch only changes when blocks are placed: every
+    # kernel waits for its predecessors at entry, so on and off agree bit for bit
+    wl = synth.tiny_workload(dtype="bf16", seed=325, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4,
+                             window=200, boundary=("uniform", 8, 190), visual=("mult", 96, 1, 3))
+    lens = synth.lengths(wl)
+    assert S.seer_set_launch_overlap(True) is True                      # on by default
+    try:
+        r_on = run_path(wl, lens)
+        assert S.seer_set_launch_overlap(False) is True
+        r_off = run_path(wl, lens)
+        assert S.seer_set_launch_overlap(True) is False
+    finally:
+        S.seer_set_launch_overlap(True)
+    for k in ("counts", "L", "cu", "kv", "xp", "y"):
+        np.testing.assert_array_equal(r_on[k], r_off[k], err_msg=k)
+    _check_path(wl, r_on)
+
+
 def test_layer_count_hook_on_full_window():
     # step-0 style: full (untruncated) window, counts fused into the gate/up epilogue
     wl = synth.tiny_workload(dtype="bf16", seed=330, d=256, n_heads=2, head_dim=128, d_ff=768, batch=3, window=160,
