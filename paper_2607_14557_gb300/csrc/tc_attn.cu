@@ -271,7 +271,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     float l = 0.f;                                // row sum
     bool ok = t < nt;
     for (int j = 0; ok && j < nkv; ++j) {
-      if (!mbar_wait(&s_full[t], j & 1, abort_flag, p.err)) { ok = false; break; }
+      // warp-uniform outcomes: the TMEM accesses that follow are warp-collective
+      if (!__all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, abort_flag, p.err))) { ok = false; break; }
       tc_fence_after();
       float s[BKV];
       {
@@ -336,7 +337,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         // (possibly non-finite) data cannot meet the zero probabilities (both
         // groups write the same zeros: each must see them before its PV)
         const int vst = j % V_STAGES;
-        if (!mbar_wait(&v_full[vst], (j / V_STAGES) & 1, abort_flag, p.err)) { ok = false; break; }
+        if (!__all_sync(0xffffffffu, mbar_wait(&v_full[vst], (j / V_STAGES) & 1, abort_flag, p.err))) { ok = false; break; }
         if (r >= valid) {
 #pragma unroll
           for (int pn = 0; pn < 2; ++pn) {
@@ -352,7 +353,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[t]);
     }
-    if (ok && nkv > 0) ok = mbar_wait(&o_done[t], 0, abort_flag, p.err);
+    if (ok && nkv > 0) ok = __all_sync(0xffffffffu, mbar_wait(&o_done[t], 0, abort_flag, p.err));
     if (ok && nkv > 0) {
       tc_fence_after();
       const float inv_l = 1.f / l;

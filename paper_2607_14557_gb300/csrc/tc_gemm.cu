@@ -238,7 +238,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
       int m, n;
       tile_coords(t, num_m, num_n, group_m, m, n);
-      if (!mbar_wait(&acc_full[acc], acc_ph, abort_flag, p.err)) break;
+      // warp-uniform outcome: the TMEM loads below are warp-collective, and
+      // after an abort the lanes of a warp could otherwise decide differently
+      if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[acc], acc_ph, abort_flag, p.err))) break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + lane_off + static_cast<uint32_t>(acc * ACC_COLS);
       if (MODE == kGemmRope) {

@@ -87,9 +87,12 @@ def test_workload0_f32_path():
     _check_path(wl, run_path(wl))
 
 
-def test_workload1_bf16_path():
+@pytest.mark.parametrize("rope_theta", [0.0, 10000.0])
+def test_workload1_bf16_path(rope_theta):
+    # 842 rows: every GEMM of the layer runs with split tiles (stream-K), the QKV
+    # projection through the rotary epilogue when rope_theta > 0
     wl = synth.workload(1)
-    _check_path(wl, run_path(wl))
+    _check_path(wl, run_path(wl, rope_theta=rope_theta))
 
 
 def test_batch_permutation_is_bit_exact():
