@@ -360,6 +360,10 @@ int seer_set_launch_overlap(int on);
  * returns accumulated milliseconds and launch counts since the last reset. */
 #define SEER_N_PHASES 11
 seer_status seer_profile_enable(int on);
+/* Restricts recording to the phases whose bit is set in phase_mask (bit i =
+ * phase i; default all).  Each recorded phase adds two events to its stream,
+ * which also keeps launch overlap from spanning that phase's boundaries. */
+seer_status seer_profile_select(uint32_t phase_mask);
 seer_status seer_profile_reset(void);
 seer_status seer_profile_read(float* ms_out, int32_t* launches_out);
 

@@ -121,6 +121,7 @@ seer_status make_map16(CUtensorMap* m, const void* base, seer_dtype dt, uint64_t
 struct Profiler {
   std::mutex mu;
   bool on = false;
+  uint32_t mask = 0xffffffffu;       // phases recorded while on
   std::vector<cudaEvent_t> pool;
   std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pending[SEER_N_PHASES];
   double ms[SEER_N_PHASES] = {};
@@ -143,7 +144,7 @@ class Phase {
  public:
   Phase(int ph, cudaStream_t st) : ph_(ph), st_(st) {
     std::lock_guard<std::mutex> lk(g_prof.mu);
-    if (!g_prof.on) return;
+    if (!g_prof.on || ((g_prof.mask >> ph) & 1u) == 0) return;
     a_ = g_prof.get();
     b_ = g_prof.get();
     if (a_ && b_) cudaEventRecord(a_, st_);
@@ -479,6 +480,12 @@ seer_status seer_selftest_wait_timeout(int limit_us, void* stream) {
 seer_status seer_profile_enable(int on) {
   std::lock_guard<std::mutex> lk(g_prof.mu);
   g_prof.on = on != 0;
+  return SEER_OK;
+}
+
+seer_status seer_profile_select(uint32_t phase_mask) {
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  g_prof.mask = phase_mask;
   return SEER_OK;
 }
 

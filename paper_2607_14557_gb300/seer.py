@@ -93,6 +93,7 @@ def lib() -> ctypes.CDLL:
             "seer_selftest_wait_timeout": [i32, vp],
             "seer_profile_enable": [i32],
             "seer_profile_reset": [],
+            "seer_profile_select": [ctypes.c_uint32],
             "seer_profile_read": [vp, vp],
         }
         for name, args in sigs.items():
@@ -260,6 +261,12 @@ def seer_check_device() -> int:
 
 def seer_profile_enable(on: bool = True):
     _check(lib().seer_profile_enable(1 if on else 0))
+
+
+def seer_profile_select(phases=None):
+    """Record only the named phases (names from PHASES; None = all)."""
+    mask = 0xFFFFFFFF if phases is None else sum(1 << PHASES.index(n) for n in phases)
+    _check(lib().seer_profile_select(mask))
 
 
 def seer_profile_reset():
