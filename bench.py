@@ -461,6 +461,11 @@ def main():
     y_full = torch.empty((T_full, d), dtype=tdt, device=dev)
 
     def timed(fn, n):
+        # each comparison starts from the same thermal state: a second idle, then
+        # two untimed calls (the truncated, padded and naive layers run back to
+        # back otherwise, and the later ones would meet a power-capped clock)
+        barrier()
+        time.sleep(1.0)
         for _ in range(2):
             fn()
         barrier()
