@@ -84,6 +84,73 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ x
   }
 }
 
+// 16-bit rows of up to 256 * VPL elements: the row is read once into
+// registers (VPL 16-byte vectors per lane, all loads in flight together), the
+// sum of squares reduced across the warp, and the row scaled from registers.
+// Two blocks per SM (at most 128 registers): 16 resident warps keep enough
+// loads in flight (35194 x 4096 rows: 6.36 TB/s, against 5.4 for the
+// two-pass streaming kernel and 4.9 at one block per SM).
+template <int IN, int OUT, int VPL>
+__global__ void __launch_bounds__(256, 2) rmsnorm_rows_kernel(const void* __restrict__ x, const void* __restrict__ g,
+                                                           void* __restrict__ y, int M_cap, const int* M_dev, int d,
+                                                           float eps, int* err) {
+  pdl_enter();
+  int M = M_cap;
+  if (M_dev != nullptr) {
+    const int md = *M_dev;
+    if (md < 0 || md > M_cap) {
+      if (blockIdx.x == 0 && threadIdx.x == 0) record_error(err, kErrRows);
+      M = md < 0 ? 0 : M_cap;
+    } else {
+      M = md;
+    }
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nwarps = gridDim.x * 8;
+  const int d8 = d / 8;
+  const uint4* xv = reinterpret_cast<const uint4*>(x);
+  const uint4* gv = reinterpret_cast<const uint4*>(g);
+  uint4* yv = reinterpret_cast<uint4*>(y);
+  for (int row = blockIdx.x * 8 + warp; row < M; row += nwarps) {
+    const size_t base8 = static_cast<size_t>(row) * d8;
+    uint4 raw[VPL];
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) {
+      const int v = lane + 32 * i;
+      raw[i] = v < d8 ? __ldg(xv + base8 + v) : make_uint4(0, 0, 0, 0);
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) {
+      const uint32_t w[4] = {raw[i].x, raw[i].y, raw[i].z, raw[i].w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float a = lo16(w[k], IN == kF16), b = hi16(w[k], IN == kF16);
+        ss = fmaf(a, a, ss);
+        ss = fmaf(b, b, ss);
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+    const float inv = rsqrtf(ss / static_cast<float>(d) + eps);
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) {
+      const int v = lane + 32 * i;
+      if (v < d8) {
+        const uint4 gq = gv[v];
+        const uint32_t w[4] = {raw[i].x, raw[i].y, raw[i].z, raw[i].w};
+        const uint32_t gw[4] = {gq.x, gq.y, gq.z, gq.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          o[k] = pack2(lo16(w[k], IN == kF16) * inv * lo16(gw[k], OUT == kF16),
+                       hi16(w[k], IN == kF16) * inv * hi16(gw[k], OUT == kF16), OUT == kF16);
+        yv[base8 + v] = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+    }
+  }
+}
+
 // Element-wise storage conversion (used once per model for f16 weight copies).
 template <int IN, int OUT>
 __global__ void convert_kernel(const void* __restrict__ src, void* __restrict__ dst, size_t n8) {
@@ -448,6 +515,18 @@ cudaError_t launch_rmsnorm(const void* x, int in_type, const void* g, void* y, i
   if (M_cap <= 0) return cudaSuccess;
   int blocks = (M_cap + 7) / 8;
   if (blocks > 65535 * 4) blocks = 65535 * 4;
+  // 16-bit rows up to 4096 wide: register-resident variant sized to the row
+  const int vpl = (d / 8 + 31) / 32;
+#define SEER_NORM_ROWS(I, O, V)                                                                                   \
+  if (in_type == I && out_type == O && vpl <= V)                                                                 \
+    return launch_kernel(rmsnorm_rows_kernel<I, O, V>, dim3(blocks), dim3(256), 0, st, x, g, y, M_cap, M_dev, d, \
+                         eps, err);
+#define SEER_NORM_16(I, O) SEER_NORM_ROWS(I, O, 4) SEER_NORM_ROWS(I, O, 8) SEER_NORM_ROWS(I, O, 16)
+  SEER_NORM_16(kBF16, kF16)
+  SEER_NORM_16(kF16, kF16)
+  SEER_NORM_16(kBF16, kBF16)
+#undef SEER_NORM_16
+#undef SEER_NORM_ROWS
 #define SEER_NORM(I, O) \
   if (in_type == I && out_type == O) return launch_kernel(rmsnorm_kernel<I, O>, dim3(blocks), dim3(256), 0, st, x, g, y, M_cap, M_dev, d, eps, err);
   SEER_NORM(kBF16, kF16)

@@ -104,8 +104,11 @@ def test_swiglu_with_count_hook(op):
 
 
 # ------------------------------------------------------------------ RMSNorm (S5, S9)
+# 16-bit rows up to 4096 wide run the register-resident kernel (4, 8 or 16 vectors
+# per lane, ragged widths masked); wider rows and fp32 the streaming one
 @pytest.mark.parametrize("x_dt,y_dt,d", [("bf16", "f16", 4096), ("f16", "f16", 256), ("bf16", "bf16", 256),
-                                         ("f32", "f32", 264)])
+                                         ("f32", "f32", 264), ("bf16", "f16", 1024), ("bf16", "f16", 3072),
+                                         ("f16", "f16", 264), ("bf16", "f16", 8192)])
 def test_rmsnorm(x_dt, y_dt, d):
     rng = _rng(8)
     M = 333
