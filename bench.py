@@ -11,8 +11,9 @@ routing + device-resident compaction, and one truncated denoising layer
 ``value``  valid tokens per second of the device-resident step (inputs in HBM);
 ``e2e``    the same metric with the host->device copy of the step's input and
            the device->host copy of its output inside the timed region;
-``--impl reference`` times the CPU oracle on a bounded sample of the same
-workload (the reference arm of this build is the oracle).
+``--impl reference`` times the CPU oracle (a plain fp64 statement of the
+method; the paper ships no code to run instead) on a bounded sample of the
+same workload.
 """
 from __future__ import annotations
 
