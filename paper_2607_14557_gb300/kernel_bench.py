@@ -4,12 +4,14 @@
     python -m paper_2607_14557_gb300.kernel_bench linear --M 35194 --N 12288 --K 4096 [--dtype f16]
     python -m paper_2607_14557_gb300.kernel_bench pack [--batch 16 --window 1024 --d 4096]
     python -m paper_2607_14557_gb300.kernel_bench scan [--batch 16 --window 1024]
+    python -m paper_2607_14557_gb300.kernel_bench norm [--M 35194 --d 4096]
 
 Each call runs the kernel `--warmup` times, then times `--reps` calls with CUDA
 events on the launching stream and prints one JSON line (ms per call and
 TFLOP/s of the algorithmic work: 4*d*sum(L^2) for attention, 2*M*N*K for a
 linear; GB/s of algorithmic bytes for pack (each kept row read and written
-once) and scan (each count read once)).  pack and scan use the lengths of the
+once) and scan (each count read once)); GB/s for norm (bf16 rows read once, f16 rows
+written once).  pack and scan use the lengths of the
 ragged 8B-layer workload (visual 729k, k in 1..5; prompt 32..128; boundary
 16..400).  Inputs are random and resident in device memory; no output is checked
 (the parity tests do that).  Used for per-kernel timings and small ncu captures.
@@ -126,6 +128,16 @@ def scan(args) -> dict:
     return {"kernel": "scan", "batch": B, "window": N, "ms": ms, "gbs": B * N * 4 / (ms * 1e-3) / 1e9}
 
 
+def norm(args) -> dict:
+    dev = torch.device("cuda", 0)
+    g = torch.Generator(device=dev).manual_seed(args.seed)
+    x = torch.randn((args.M, args.d), device=dev, generator=g).to(torch.bfloat16)
+    gain = torch.ones(args.d, device=dev, dtype=torch.float16)
+    y = torch.empty((args.M, args.d), device=dev, dtype=torch.float16)
+    ms = _time(lambda: S.seer_rmsnorm(x, "bf16", gain, y, "f16", args.M, None, args.d, 1e-5), args.warmup, args.reps)
+    return {"kernel": "norm", "M": args.M, "d": args.d, "ms": ms, "gbs": args.M * args.d * 4 / (ms * 1e-3) / 1e9}
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     sub = ap.add_subparsers(dest="kernel", required=True)
@@ -148,12 +160,15 @@ def main(argv=None):
     ps = sub.add_parser("scan")
     ps.add_argument("--batch", type=int, default=16)
     ps.add_argument("--window", type=int, default=1024)
-    for q in (pp, ps):
+    pn = sub.add_parser("norm")
+    pn.add_argument("--M", type=int, default=35194)
+    pn.add_argument("--d", type=int, default=4096)
+    for q in (pp, ps, pn):
         q.add_argument("--warmup", type=int, default=3)
         q.add_argument("--reps", type=int, default=10)
         q.add_argument("--seed", type=int, default=0)
     args = ap.parse_args(argv)
-    res = {"attention": attention, "linear": linear, "pack": pack, "scan": scan}[args.kernel](args)
+    res = {"attention": attention, "linear": linear, "pack": pack, "scan": scan, "norm": norm}[args.kernel](args)
     assert S.seer_check_device() == 0, "a kernel recorded a device-side error"
     print(json.dumps(res), flush=True)
 
