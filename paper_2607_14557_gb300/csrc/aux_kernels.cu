@@ -1,5 +1,6 @@
 // Memory- and latency-bound kernels of the hot path:
-//   rmsnorm          pre-attention / pre-MLP normalisation (one warp per row)
+//   rmsnorm          pre-attention / pre-MLP normalisation (one warp per row;
+//                    16-bit rows up to 4096 wide held in registers, else two passes)
 //   snr_scan         Seer Sec. 3.3 boundary criterion, one warp per sequence
 //   pack_route       Seer Sec. 3.4-3.5: micro-bucket routing (Eq. 4) fused
 //                    with device-resident compaction and the pinned control word
