@@ -290,7 +290,38 @@ def run_stack(args, wl, world, rank, local):
         evc[3].record(stream)
         torch.cuda.synchronize()
     assert S.seer_check_device() == 0
-    assert S.seer_check_device() == 0
+
+    # ---- end to end: one generation through the public API from pinned host
+    # memory: upload the step-0 input, step 0 + route/pack, the 63 truncated steps,
+    # then download the last step's packed output rows and L*
+    e2e = None
+    if not args.no_e2e:
+        x_host = torch.from_numpy(x_np).to(torch.bfloat16).pin_memory()
+        x_dev = torch.empty_like(x_full)
+        out_host = torch.empty((T_full, wl.d), dtype=torch.bfloat16).pin_memory()
+        L_host = torch.empty(wl.batch, dtype=torch.int32).pin_memory()
+        torch.cuda.synchronize()
+        a_e, b_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t_e = time.perf_counter()
+        a_e.record(stream)
+        x_dev.copy_(x_host, non_blocking=True)
+        stack.step0(x_dev, cu_full, resp, ctx, stream)
+        r_e = stack.path.route()
+        g_e = stack.truncated_graph(r_e["capacity"])
+        for _ in range(n_steps - 1):
+            g_e.replay()
+        out_dev = stack.buf[(wl.n_layers - 1) % 2]
+        out_host[:r_e["total"]].copy_(out_dev[:r_e["total"]], non_blocking=True)
+        L_host.copy_(stack.path.L_star, non_blocking=True)
+        b_e.record(stream)
+        torch.cuda.synchronize()
+        ms_e2e = max(a_e.elapsed_time(b_e), (time.perf_counter() - t_e) * 1e3)
+        tok_e = (T_full + (n_steps - 1) * T_valid) * wl.n_layers
+        e2e = {"value": tok_e / (ms_e2e * 1e-3), "unit": "tokens/s", "ms_per_generation": ms_e2e,
+               "h2d_bytes_per_step": x_host.numel() * x_host.element_size() / n_steps,
+               "d2h_bytes_per_step": (r_e["total"] * wl.d * 2 + wl.batch * 4) / n_steps,
+               "note": "one generation (64 steps): the input uploaded once, the last step's rows downloaded once"}
+        assert S.seer_check_device() == 0
     ms0 = ev[0].elapsed_time(ev[1])
     ms_rest = ev[1].elapsed_time(ev[2])
     ms_pad = ev[2].elapsed_time(ev[3])
@@ -339,6 +370,7 @@ def run_stack(args, wl, world, rank, local):
                      "bound": "tensor", "achieved": tflops_rest, "peak": pk["bf16_tflops_sustained"],
                      "unit": "TFLOP/s", "frac": tflops_rest / pk["bf16_tflops_sustained"], "traffic": None,
                      "peak_source": f"{src} bf16 dense, sustained (a {ms_rest / 1e3:.0f} s region under the power cap)"},
+        "e2e": e2e,
         "gpu_launches": nl * 8 * (2 * n_steps) + 3 + (nl * 8 + 4)
                         + (nl * 8 + 3) + nl * 13 + (n_steps - 2) * (2 + nl * 9), "clocks": clk.summary(),
         "peak_source": src,
