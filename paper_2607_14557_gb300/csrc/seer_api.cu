@@ -3,6 +3,7 @@
 // arithmetic runs in the kernels of tc_gemm.cu, tc_attn.cu, simt.cu and
 // aux_kernels.cu.
 #include <cudaTypedefs.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <atomic>
 #include <chrono>
@@ -139,10 +140,18 @@ struct Profiler {
 };
 Profiler g_prof;
 
-// Records a pair of events around one kernel launch when profiling is on.
+// NVTX range names of the phases (same order as seer_profile_read).
+const char* const kPhaseNames[SEER_N_PHASES] = {"seer:detect_gemm", "seer:snr_scan", "seer:pack",  "seer:norm1",
+                                                 "seer:qkv",         "seer:attention", "seer:o_proj", "seer:norm2",
+                                                 "seer:gate_up",     "seer:down",      "seer:kv_cache"};
+
+// Marks one kernel launch: an NVTX range on the host timeline (a no-op unless
+// a tool such as nsys or ncu --nvtx is attached), and, when profiling is on,
+// a pair of CUDA events on the launch's stream.
 class Phase {
  public:
   Phase(int ph, cudaStream_t st) : ph_(ph), st_(st) {
+    nvtxRangePushA(kPhaseNames[ph]);
     std::lock_guard<std::mutex> lk(g_prof.mu);
     if (!g_prof.on || ((g_prof.mask >> ph) & 1u) == 0) return;
     a_ = g_prof.get();
@@ -150,6 +159,7 @@ class Phase {
     if (a_ && b_) cudaEventRecord(a_, st_);
   }
   ~Phase() {
+    nvtxRangePop();
     if (!a_ || !b_) return;
     cudaEventRecord(b_, st_);
     std::lock_guard<std::mutex> lk(g_prof.mu);
