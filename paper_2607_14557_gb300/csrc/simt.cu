@@ -11,7 +11,8 @@ namespace seer {
 namespace {
 
 constexpr int TB = 64;   // output tile (rows and columns)
-constexpr int TK = 16;
+constexpr int TK = 32;
+constexpr int LPT = TB * TK / 256;   // elements of each operand tile a thread loads per k-step
 
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)); }
 
@@ -61,16 +62,32 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const float* __restrict_
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
   float acc0[4][4] = {}, acc1[4][4] = {};
 
-  for (int k0 = 0; k0 < p.K; k0 += TK) {
-    for (int i = threadIdx.x; i < TB * TK; i += 256) {
-      const int r = i / TK, k = i % TK;
-      const int kk = k0 + k;
-      As[k][r] = (r < rows_here && kk < p.K) ? A[static_cast<size_t>(row_base + r) * p.K + kk] : 0.f;
+  // the next k-step's operands are loaded into registers while the current
+  // one is multiplied out of shared memory
+  float ra[LPT], rb0[LPT], rb1[LPT];
+  auto load = [&](int k0) {
+#pragma unroll
+    for (int e = 0; e < LPT; ++e) {
+      const int i = threadIdx.x + 256 * e;
+      const int r = i / TK, kk = k0 + i % TK;
+      ra[e] = (r < rows_here && kk < p.K) ? A[static_cast<size_t>(row_base + r) * p.K + kk] : 0.f;
       const int c = col_base + r;
-      Bs0[k][r] = (c < p.N && kk < p.K) ? B0[static_cast<size_t>(c) * p.K + kk] : 0.f;
-      if (TWO) Bs1[k][r] = (c < p.N && kk < p.K) ? B1[static_cast<size_t>(c) * p.K + kk] : 0.f;
+      rb0[e] = (c < p.N && kk < p.K) ? B0[static_cast<size_t>(c) * p.K + kk] : 0.f;
+      if (TWO) rb1[e] = (c < p.N && kk < p.K) ? B1[static_cast<size_t>(c) * p.K + kk] : 0.f;
+    }
+  };
+  load(0);
+  for (int k0 = 0; k0 < p.K; k0 += TK) {
+#pragma unroll
+    for (int e = 0; e < LPT; ++e) {
+      const int i = threadIdx.x + 256 * e;
+      const int r = i / TK, k = i % TK;
+      As[k][r] = ra[e];
+      Bs0[k][r] = rb0[e];
+      if (TWO) Bs1[k][r] = rb1[e];
     }
     __syncthreads();
+    if (k0 + TK < p.K) load(k0 + TK);
 #pragma unroll
     for (int k = 0; k < TK; ++k) {
       float a[4], b0[4], b1[4];
@@ -169,25 +186,50 @@ __global__ void __launch_bounds__(256) simt_attn_kernel(const float* __restrict_
   }
   const float scale = 1.0f / sqrtf(static_cast<float>(dh));
   float m = -INFINITY, l = 0.f;
-  for (int kidx = 0; kidx < kvL; ++kidx) {
-    const float* kvrow = kvsrc + static_cast<size_t>(kv0 + kidx) * p.ld_kv;
-    const float* krow = kvrow + p.xk0 + h * dh;
-    const float* vrow = kvrow + p.xv0 + h * dh;
-    float part = 0.f;
-    for (int i = 0; i < per; ++i) {
-      const int c = lane + 32 * i;
-      if (c < dh) part = fmaf(q[i], krow[c], part);
+  // keys in chunks of KC: the chunk's loads are all in flight together and its
+  // KC warp reductions are independent, then one online-softmax update
+  constexpr int KC = 8;
+  for (int k0 = 0; k0 < kvL; k0 += KC) {
+    float kv_k[KC][4], kv_v[KC][4], sc[KC];
+#pragma unroll
+    for (int j = 0; j < KC; ++j) {
+      const bool valid = k0 + j < kvL;
+      const float* kvrow = kvsrc + static_cast<size_t>(kv0 + (valid ? k0 + j : 0)) * p.ld_kv;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int c = lane + 32 * i;
+        const bool in = valid && i < per && c < dh;
+        kv_k[j][i] = in ? kvrow[p.xk0 + h * dh + c] : 0.f;
+        kv_v[j][i] = in ? kvrow[p.xv0 + h * dh + c] : 0.f;
+      }
     }
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
-    const float sc = part * scale;
-    const float m_new = fmaxf(m, sc);
+    for (int j = 0; j < KC; ++j) {
+      float part = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) part = fmaf(q[i], kv_k[j][i], part);
+      sc[j] = part;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+      for (int j = 0; j < KC; ++j) sc[j] += __shfl_xor_sync(0xffffffffu, sc[j], off);
+    float m_new = m;
+#pragma unroll
+    for (int j = 0; j < KC; ++j) {
+      sc[j] = k0 + j < kvL ? sc[j] * scale : -INFINITY;
+      m_new = fmaxf(m_new, sc[j]);
+    }
     const float alpha = expf(m - m_new);
-    const float pr = expf(sc - m_new);
-    l = l * alpha + pr;
-    for (int i = 0; i < per; ++i) {
-      const int c = lane + 32 * i;
-      o[i] = o[i] * alpha + (c < dh ? pr * vrow[c] : 0.f);
+    l *= alpha;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) o[i] *= alpha;
+#pragma unroll
+    for (int j = 0; j < KC; ++j) {
+      const float pr = expf(sc[j] - m_new);
+      l += pr;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) o[i] = fmaf(pr, kv_v[j][i], o[i]);
     }
     m = m_new;
   }
