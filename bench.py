@@ -179,6 +179,39 @@ def oracle_sample(wl):
                       f"window + one truncated layer, fp64 numpy"
 
 
+def reference_config(wl, world, args) -> dict:
+    """The ``config`` of this workload as our arm reports it, computed on the
+    host from the synthetic lengths and the oracle's routing (the planted
+    boundaries give L* = b + 1, which the GPU detection reproduces exactly)."""
+    import oracle
+    lens = synth.lengths(wl)
+    L = (lens.boundary + 1).astype(np.int64)
+    tau = 0.2
+    seg, kv, cu = oracle.segment_layout(lens.ctx, L, wl.window, tau)
+    T_full, T_valid, T_exec = int(lens.full.sum()), int(kv.sum()), int(cu[-1])
+    groups = [{"bucket": g["bucket"], "members": len(g["members"]), "path": g["path"],
+               "rho": int(np.floor(g["rho"] * 1e6)) / 1e6} for g in oracle.route(L, wl.window, tau)]
+    pad = int(sum(g["bucket"] * len(g["members"]) - int(L[g["members"]].sum())
+                  for g in oracle.route(L, wl.window, tau) if g["path"] == oracle.PATH_STATIC))
+    d, F = wl.d, wl.d_ff
+    if wl.index == 3:
+        return {"workload": f"{wl.name} (workload 3): {wl.n_layers} layers x {wl.steps} denoising steps, batch "
+                            f"{wl.batch}, window {wl.window}, d {d}, F {F}; tokens counted once per layer and step",
+                "tokens_full": T_full, "tokens_valid": T_valid, "tokens_executed": T_exec, "L_star": L.tolist(),
+                "route": {"groups": groups, "capacity": graph_capacity(T_exec)},
+                "l2": "inputs larger than L2 (weights %.1f GB)" % (wl.n_layers * (4 * d * d + 3 * d * F) * 2 / 1e9),
+                "launch_overlap": args.launch_overlap}
+    es = 2 if wl.dtype == "bf16" else 4
+    return {"workload": f"{wl.name} (workload {wl.index}): batch {wl.batch}, window {wl.window}, "
+                        f"d {d}, heads {wl.n_heads}x{wl.head_dim}, F {F}",
+            "batch": wl.batch, "window": wl.window, "tokens_full": T_full, "tokens_valid": T_valid,
+            "tokens_executed": T_exec, "L_star": L.tolist(),
+            "l2": "inputs larger than L2 (x_full %.0f MB, weights %.0f MB)" % (T_full * d * es / 1e6,
+                                                                              (4 * d * d + 3 * d * F) * 2 / 1e6),
+            "route": {"groups": groups, "pad_rows": pad, "capacity": graph_capacity(T_exec)},
+            "parallelism": f"replicas x{world}", "launch_overlap": args.launch_overlap}
+
+
 def run_reference(args, wl, rank, world):
     if rank != 0:
         return
@@ -195,7 +228,7 @@ def run_reference(args, wl, rank, world):
     line = {"metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": wl.name, "index": wl.index},
+            "config": reference_config(wl, world, args),
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
