@@ -247,6 +247,10 @@ def run_stack(args, wl, world, rank, local):
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    from paper_2607_14557_gb300 import replicas as R
     detect_layer = 3
     lens = synth.lengths(wl)
     x_np, cu_full_np, resp_np = synth.hidden_full(wl, lens)
@@ -282,7 +286,7 @@ def run_stack(args, wl, world, rank, local):
     d, F, nl = wl.d, wl.d_ff, wl.n_layers
 
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
-    torch.cuda.synchronize()
+    R.barrier(dev)
     with ClockSampler(local) as clk:
         ev[0].record(stream)
         stack.step0(x_full, cu_full, resp, ctx, stream)
@@ -367,7 +371,9 @@ def run_stack(args, wl, world, rank, local):
     fl_trunc = layer_flops(seg, kv, d, F) * nl
     fl_valid = layer_flops(kv, kv, d, F) * nl
     tok_layers = (T_full + (n_steps - 1) * T_valid) * nl
-    value = tok_layers / (ms_seer * 1e-3)
+    # replicas: every rank runs its own batch; the job's rate is all ranks'
+    # token-layers over the slowest rank's time
+    value = R.sum_over_ranks(tok_layers, dev) / (R.max_over_ranks(ms_seer, dev) * 1e-3)
     pk, src = peaks()
     tflops_rest = fl_trunc * (n_steps - 1) / (ms_rest * 1e-3) / 1e12
     line = {
