@@ -345,6 +345,17 @@ def test_pack_route_untruncated_is_identity_layout():
     _pack_case("bf16", ctx, [N, N, N], N, 256, seed=3)
 
 
+@pytest.mark.parametrize("B,tau_pad,bucket_min", [(64, 0.2, 8), (256, 0.2, 8), (256, -1.0, 1), (256, 0.9, 64)])
+def test_pack_route_large_batches(B, tau_pad, bucket_min):
+    # the routing ablation's batch sizes: every block recomputes the route of all
+    # B sequences in shared memory; groups, layout, control word and rows exact
+    rng = _rng(40 + B)
+    N = 1024
+    ctx = list(map(int, rng.integers(0, 3000, B)))
+    L = list(map(int, rng.integers(1, N + 1, B)))
+    _pack_case("bf16", ctx, L, N, 64, tau_pad=tau_pad, seed=41 + B, bucket_min=bucket_min)
+
+
 @pytest.mark.parametrize("bucket_min", [1, 16, 64, 1024])
 def test_pack_route_bucket_set_variants(bucket_min):
     # the smallest micro-bucket moves the group boundaries (routing ablation)
