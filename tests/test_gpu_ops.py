@@ -200,6 +200,27 @@ def test_snr_scan_golden_bit_exact():
         assert (int(I.item()), int(L.item())) == (case["i_star"], case["L_star"]), case["name"]
 
 
+@pytest.mark.parametrize("B,N", [(256, 1024), (3, 20000)])
+def test_snr_scan_large_shapes_match_oracle_exactly(B, N):
+    # many sequences (one warp each), and a window longer than the shared-memory
+    # staging of the counts (the scan then reads them from global memory)
+    rng = _rng(50 + N)
+    F = 12288
+    counts = rng.integers(0, 100, size=(B, N))
+    for b in range(B):
+        j = int(rng.integers(1, N - 3))
+        counts[b, j:] += int(rng.integers(0, 3000))        # a jump below tau_jump * F (369) is no boundary
+    counts[0, :] = 0                                       # no jump at all: L* = N
+    p = S.make_params(0.0, 0.03, 0.6, 3)
+    L = torch.empty(B, dtype=torch.int32, device=cuda())
+    I = torch.empty(B, dtype=torch.int32, device=cuda())
+    S.seer_snr_scan(i32(counts.ravel()), B, N, F, p, L, I)
+    i_ref, L_ref = oracle.snr_boundaries(counts, F, 0.03, 0.6, 3)
+    np.testing.assert_array_equal(I.cpu().numpy(), i_ref)
+    np.testing.assert_array_equal(L.cpu().numpy(), L_ref)
+    assert L_ref[0] == N and (L_ref[1:] < N).any()
+
+
 def test_snr_scan_random_matches_oracle_exactly():
     rng = _rng(14)
     B, N, F = 37, 300, 768
