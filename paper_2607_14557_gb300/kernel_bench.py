@@ -5,11 +5,12 @@
     python -m paper_2607_14557_gb300.kernel_bench pack [--batch 16 --window 1024 --d 4096]
     python -m paper_2607_14557_gb300.kernel_bench scan [--batch 16 --window 1024]
     python -m paper_2607_14557_gb300.kernel_bench norm [--M 35194 --d 4096]
+    python -m paper_2607_14557_gb300.kernel_bench swiglu --M 35194 --F 12288 --K 4096 [--dtype f16]
 
 Each call runs the kernel `--warmup` times, then times `--reps` calls with CUDA
 events on the launching stream and prints one JSON line (ms per call and
 TFLOP/s of the algorithmic work: 4*d*sum(L^2) for attention, 2*M*N*K for a
-linear; GB/s of algorithmic bytes for pack (each kept row read and written
+linear, 4*M*F*K for the gate/up GEMM with its SwiGLU epilogue; GB/s of algorithmic bytes for pack (each kept row read and written
 once) and scan (each count read once)); GB/s for norm (bf16 rows read once, f16 rows
 written once).  pack and scan use the lengths of the
 ragged 8B-layer workload (visual 729k, k in 1..5; prompt 32..128; boundary
@@ -86,6 +87,20 @@ def linear(args) -> dict:
             "tflops": 2.0 * args.M * args.N * args.K / (ms * 1e-3) / 1e12}
 
 
+def swiglu(args) -> dict:
+    dev = torch.device("cuda", 0)
+    tdt = {"f16": torch.float16, "bf16": torch.bfloat16}[args.dtype]
+    g = torch.Generator(device=dev).manual_seed(args.seed)
+    a = (0.5 * torch.randn((args.M, args.K), device=dev, generator=g)).to(tdt)
+    wg = (0.02 * torch.randn((args.F, args.K), device=dev, generator=g)).to(tdt)
+    wu = (0.02 * torch.randn((args.F, args.K), device=dev, generator=g)).to(tdt)
+    act = torch.empty((args.M, args.F), device=dev, dtype=tdt)
+    ms = _time(lambda: S.seer_swiglu(a, wg, wu, args.dtype, act, args.dtype, args.M, None, args.F, args.K),
+               args.warmup, args.reps)
+    return {"kernel": "swiglu", "M": args.M, "F": args.F, "K": args.K, "dtype": args.dtype, "ms": ms,
+            "tflops": 4.0 * args.M * args.F * args.K / (ms * 1e-3) / 1e12}
+
+
 def _ragged_lengths(batch, seed):
     rng = np.random.default_rng(seed)
     ctx = 729 * rng.integers(1, 6, batch) + rng.integers(32, 129, batch)
@@ -148,7 +163,11 @@ def main(argv=None):
     pl.add_argument("--M", type=int, default=35194)
     pl.add_argument("--N", type=int, default=12288)
     pl.add_argument("--K", type=int, default=4096)
-    for p in (pa, pl):
+    pw = sub.add_parser("swiglu")
+    pw.add_argument("--M", type=int, default=35194)
+    pw.add_argument("--F", type=int, default=12288)
+    pw.add_argument("--K", type=int, default=4096)
+    for p in (pa, pl, pw):
         p.add_argument("--dtype", default="f16", choices=["f16", "bf16"])
         p.add_argument("--warmup", type=int, default=3)
         p.add_argument("--reps", type=int, default=10)
@@ -168,7 +187,7 @@ def main(argv=None):
         q.add_argument("--reps", type=int, default=10)
         q.add_argument("--seed", type=int, default=0)
     args = ap.parse_args(argv)
-    res = {"attention": attention, "linear": linear, "pack": pack, "scan": scan, "norm": norm}[args.kernel](args)
+    res = {"attention": attention, "linear": linear, "pack": pack, "scan": scan, "norm": norm, "swiglu": swiglu}[args.kernel](args)
     assert S.seer_check_device() == 0, "a kernel recorded a device-side error"
     print(json.dumps(res), flush=True)
 
