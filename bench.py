@@ -63,20 +63,31 @@ def peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
+def code_digest(paths) -> str:
+    """SHA-1 of the code in `paths` (files relative to the repository root) with
+    `//` comments, trailing blanks and empty lines removed, so that editing a
+    comment does not invalidate a capture."""
+    import hashlib
+    import re
+    h = hashlib.sha1()
+    for s in paths:
+        with open(os.path.join(ROOT, s)) as f:
+            for line in f:
+                code = re.sub(r"//.*$", "", line).rstrip()
+                if code:
+                    h.update(code.encode() + b"\n")
+    return h.hexdigest()
+
+
 def measured_traffic(workload: int, kernel: str):
     """DRAM bytes per launch of `kernel` from the committed ncu capture of this
-    workload, or None when the kernel sources changed since that capture."""
-    import hashlib
+    workload, or None when the kernel code changed since that capture."""
     path = os.path.join(ROOT, "profiles", f"traffic_workload{workload}.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         doc = json.load(f)
-    h = hashlib.sha1()
-    for s in doc["sources"]:
-        with open(os.path.join(ROOT, s), "rb") as f:
-            h.update(f.read())
-    if h.hexdigest() != doc["sources_sha1"] or kernel not in doc["kernels"]:
+    if code_digest(doc["sources"]) != doc.get("sources_code_sha1") or kernel not in doc["kernels"]:
         return None
     return doc["kernels"][kernel]["traffic_bytes"]
 

@@ -14,7 +14,9 @@
 //               32 x 32 output chunks staged in shared memory and written by
 //               TMA stores marked L2 evict-first (a tile whose rows run past
 //               the device row count stores its valid rows lane by lane).
-// The epilogue of tile t overlaps the main loop of tile t+1.
+// The epilogue of tile t overlaps the main loop of tile t+1.  Every CTA waits
+// for the previous kernel of the stream at entry (griddepcontrol.wait) and
+// lets the next kernel launch once its last MMAs are issued.
 //
 // Epilogues (Sec. 3.1 Eq. 2 projections; Sec. 3.2 sparsity hook):
 //   Store     C = A B^T                                    (QKV projection)
