@@ -55,8 +55,9 @@ struct AttnParams {
   int head_dim;
   void* out;              // [T, H*dh]
   int ldo;                // elements
-  const int4* work;       // schedule: (b, h, q-tile, 0)
-  const int* work_count;
+  const int4* work;       // schedule: (b, h, first q-tile, q-tiles)
+  const int* work_count;  // units in `work`
+  int* work_next;         // next unit to hand out (zeroed by the schedule kernel)
   int* err;
 };
 
@@ -70,8 +71,12 @@ int tc_gemm_group_m(long b_bytes, long a_tile_bytes);
 cudaError_t launch_tc_gemm(int mode, const CUtensorMap& mA, const CUtensorMap& mB0, const CUtensorMap& mB1,
                            const CUtensorMap& mC, const GemmParams& p, int num_sms, cudaStream_t st);
 int tc_attn_smem_bytes();
+// grid: persistent CTAs (at most one per SM); they take the units of the
+// schedule from p.work_next until *p.work_count are done
 cudaError_t launch_tc_attn(const CUtensorMap& mQ, const CUtensorMap& mKV, const AttnParams& p, int grid, bool f16,
                            cudaStream_t st);
+// writes the units to work, their number to work_count[0] and zeroes
+// work_count[1] (the attention kernel's unit counter)
 cudaError_t launch_attn_schedule(const int* cu, const int* cu_kv, const int* kv_len, int B, int n_heads, int T_cap,
                                  int4* work, int* work_count, int max_units, int* err, cudaStream_t st);
 

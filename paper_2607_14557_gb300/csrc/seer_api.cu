@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 #include <nvtx3/nvToolsExt.h>
 
+#include <algorithm>
 #include <atomic>
 #include <chrono>
 #include <cmath>
@@ -423,13 +424,16 @@ seer_status do_attention(const void* qkv, void* o, seer_dtype dt, const int32_t*
     int* count = reinterpret_cast<int*>(static_cast<uint8_t*>(sched) + align256(static_cast<size_t>(max_units) * sizeof(int4)));
     p.work = work;
     p.work_count = count;
+    p.work_next = count + 1;
     CUtensorMap m, mkv;
     SEER_TRY(make_map16(&m, qkv, dt, T_cap, 3 * H * dh, 3 * H * dh, 128));
     if (kvs.kv) SEER_TRY(make_map16(&mkv, kvs.kv, dt, kvs.T_kv_cap > 0 ? kvs.T_kv_cap : 1, kvs.ld, kvs.ld, 128));
     Phase ph(PH_ATTN, st);
     SEER_CUDA(launch_attn_schedule(cu, p.cu_kv, kv_len, B, H, T_cap, work, count, max_units, di->err, st),
               "attn schedule");
-    SEER_CUDA(launch_tc_attn(m, kvs.kv ? mkv : m, p, max_units, dt == SEER_F16, st), "tc_attn launch");
+    // persistent: one CTA per SM (at most one per unit)
+    SEER_CUDA(launch_tc_attn(m, kvs.kv ? mkv : m, p, std::min(max_units, di->num_sms), dt == SEER_F16, st),
+              "tc_attn launch");
   } else {
     if (dh > 128 || dh % 4 != 0) return fail(SEER_ERR_UNSUPPORTED, "fp32 attention needs head_dim <= 128, %% 4 == 0");
     if (T_cap == 0) return SEER_OK;

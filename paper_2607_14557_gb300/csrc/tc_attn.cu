@@ -5,10 +5,17 @@
 // the first kv_len[b] rows of the same segment, with no causal mask; rows
 // beyond kv_len (bucket padding of the static path) are never keys.
 //
-// One CTA per (segment, head, pair of 128-query tiles); 384 threads:
-//   warp 0     TMA producers: both Q tiles once, then K_j (lane 0, 2-deep
-//              ring) and V_j (lane 1, 2-deep ring), 128 keys x 128 dims with
-//              128-byte swizzle;
+// Work unit = (segment, head, pair of 128-query tiles).  Persistent CTAs, one
+// per SM (384 threads), take units from a global counter in schedule order
+// (longest segment first) until none are left; every ring and barrier phase
+// runs on across units, so a unit's Q / K loads and first QK^T overlap the
+// previous unit's last PV and epilogue (a CTA per unit paid ~3.4 us of
+// setup and teardown per unit, the persistent loop ~0.3 us).
+//   warp 0     TMA producers: lane 0 takes the next unit (atomic counter) and
+//              publishes its index in a 4-entry shared ring, loads the unit's
+//              Q tiles once both issuers are done with the previous ones, and
+//              its K_j (2-deep ring); lane 1 loads V_j (2-deep ring); 128 keys
+//              x 128 dims with 128-byte swizzle;
 //   warps 1-2  TMEM allocator (warp 1) and one MMA issuer per query tile t:
 //              O_t += P_t,j-1 V_j-1 (P from tensor memory, V an MN-major
 //              shared operand), then S_t,j = Q_t K_j^T (both from shared
@@ -18,7 +25,13 @@
 //              tile's MMA stream (the pipe's issue queue is shallow); a turn
 //              token passed between them keeps the rounds in ping-pong order
 //              (tile 0's PV + QK^T, then tile 1's), so the two softmax groups
-//              work in alternation instead of in lock step;
+//              work in alternation instead of in lock step.  The issuer sits
+//              on each round's critical path (softmax -> P -> next MMAs), so
+//              its steady-state loop carries no per-round conditions: the
+//              first (QK^T only) and last (PV only) rounds are peeled, and
+//              ring positions are unsigned counters (stage = c % 2, phase =
+//              c / 2 % 2).  A tile idle in a unit (odd tile count) only
+//              releases the Q, K and V stages it would have used;
 //   warps 4-7  softmax of query tile 0, warps 8-11 of tile 1: one thread per
 //              query row holds the row's 128 scores, so no exchange between
 //              threads is needed.  While one group exponentiates its tile,
@@ -26,8 +39,8 @@
 // Online softmax in the log2 domain with lazy rescaling: O_t is rescaled in
 // tensor memory only when the running max grows by more than 2^8.
 // Tensor memory (512 columns): S_0 | S_1 | O_0 | O_1, P_t packed into the
-// first 64 columns of S_t.
-// The schedule kernel orders work units longest segment first.
+// first 64 columns of S_t; a unit's first PV waits until the softmax warps
+// have read the previous unit's O_t out.
 #include <math.h>
 
 #include "common.cuh"
@@ -55,6 +68,11 @@ constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t TM_S = 0;                // S_t at TM_S + 128 t
 constexpr uint32_t TM_O = 256;              // O_t at TM_O + 128 t
 constexpr float RESCALE_THRESHOLD = 8.0f;   // log2 units
+constexpr int U_SLOTS = 4;                  // unit indices published ahead
+constexpr int U_READERS = 1 + NT + 4 * NT;   // V lane, NT issuers, 4 softmax warps per tile
+// barriers (8 bytes each), the unit ring, the TMEM base and the abort flag
+static_assert(8 * (2 + 2 * K_STAGES + 2 * V_STAGES + 5 * NT + 2 * U_SLOTS) + 4 * U_SLOTS + 8 <= 256,
+              "barrier block");
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -111,35 +129,66 @@ __device__ __forceinline__ void row_probs(const float* s, float scale_log2, floa
   }
 }
 
+struct Unit {
+  int b, h, qt0, nt, seq0, L, kv0, kvL, q0, nkv, xq, xk, xv;
+};
+
+__device__ __forceinline__ Unit decode_unit(const AttnParams& p, int u) {
+  Unit d;
+  const int4 wk = p.work[u];
+  d.b = wk.x;
+  d.h = wk.y;
+  d.qt0 = wk.z;
+  d.nt = wk.w;
+  d.seq0 = p.cu[d.b];
+  d.L = p.cu[d.b + 1] - d.seq0;
+  d.kv0 = p.cu_kv ? p.cu_kv[d.b] : d.seq0;
+  d.kvL = p.kv_len ? p.kv_len[d.b] : (p.cu_kv ? p.cu_kv[d.b + 1] - d.kv0 : d.L);
+  d.q0 = d.seq0 + d.qt0 * BQ;
+  d.nkv = (d.kvL + BKV - 1) / BKV;
+  d.xq = d.h * DH;
+  d.xk = p.xk0 + d.h * DH;
+  d.xv = p.xv0 + d.h * DH;
+  return d;
+}
+
+// Unit index of this CTA's i-th unit, read from the shared ring (-1: no more
+// units or an abort); `arrive` releases the slot for this reader.
+__device__ __forceinline__ int read_unit(uint64_t* u_full, uint64_t* u_empty, const int* unit_slot, int i,
+                                         volatile int* abort, int* err, bool arrive) {
+  const int s = i % U_SLOTS;
+  if (!mbar_wait(&u_full[s], (i / U_SLOTS) & 1, abort, err)) return -1;
+  const int u = unit_slot[s];
+  if (arrive) mbar_arrive(&u_empty[s]);
+  return u;
+}
+
 template <bool F16>
 __global__ void __launch_bounds__(THREADS, 1)
     tc_attn_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mKV, const AttnParams p) {
   pdl_enter();
-  const int u = blockIdx.x;
-  if (u >= *p.work_count) return;
-  const int4 wk = p.work[u];
-  const int b = wk.x, h = wk.y, qt0 = wk.z, nt = wk.w;   // query tiles qt0 .. qt0 + nt - 1
-  const int seq0 = p.cu[b];
-  const int L = p.cu[b + 1] - seq0;
-  const int kv0 = p.cu_kv ? p.cu_kv[b] : seq0;  // first K/V row of the segment
-  const int kvL = p.kv_len ? p.kv_len[b] : (p.cu_kv ? p.cu_kv[b + 1] - kv0 : L);
-  const int q0 = seq0 + qt0 * BQ;
-  const int nkv = (kvL + BKV - 1) / BKV;
-  const int xq = h * DH, xk = p.xk0 + h * DH, xv = p.xv0 + h * DH;
+  const int count = *p.work_count;
+  if (static_cast<int>(blockIdx.x) >= count) return;
+  const int G = gridDim.x;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;               // [K_STAGES]
+  uint64_t* q_empty = bars + 1;              // both issuers are done with the Q tiles of a unit
+  uint64_t* k_full = bars + 2;               // [K_STAGES]
   uint64_t* k_empty = k_full + K_STAGES;     // [K_STAGES]
   uint64_t* v_full = k_empty + K_STAGES;     // [V_STAGES]
   uint64_t* v_empty = v_full + V_STAGES;     // [V_STAGES]
   uint64_t* s_full = v_empty + V_STAGES;     // [NT] S_t,j written (and O_t += P_t,j-1 V done)
   uint64_t* p_full = s_full + NT;            // [NT] P_t,j in tensor memory (O_t rescaled)
-  uint64_t* o_done = p_full + NT;            // [NT] last PV of tile t complete
-  uint64_t* turn = o_done + NT;              // [NT] issuer t may enqueue its next round
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(turn + NT);
+  uint64_t* o_done = p_full + NT;            // [NT] last PV of tile t of a unit complete
+  uint64_t* o_free = o_done + NT;            // [NT] O_t of a unit read out by the softmax warps
+  uint64_t* turn = o_free + NT;              // [NT] issuer t may enqueue its next round
+  uint64_t* u_full = turn + NT;              // [U_SLOTS] unit index published
+  uint64_t* u_empty = u_full + U_SLOTS;      // [U_SLOTS] unit index read by every role
+  int* unit_slot = reinterpret_cast<int*>(u_empty + U_SLOTS);   // [U_SLOTS]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(unit_slot + U_SLOTS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -147,19 +196,25 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
+    mbar_init(q_empty, NT);
     for (int i = 0; i < K_STAGES; ++i) {
       mbar_init(&k_full[i], 1);
-      mbar_init(&k_empty[i], nt);      // one commit per tile issuer
+      mbar_init(&k_empty[i], NT);      // one commit (or, for an idle tile, one arrive) per issuer
     }
     for (int i = 0; i < V_STAGES; ++i) {
       mbar_init(&v_full[i], 1);
-      mbar_init(&v_empty[i], nt);
+      mbar_init(&v_empty[i], NT);
     }
     for (int t = 0; t < NT; ++t) {
       mbar_init(&s_full[t], 1);
       mbar_init(&p_full[t], 4);
       mbar_init(&o_done[t], 1);
+      mbar_init(&o_free[t], 4);
       mbar_init(&turn[t], 1);
+    }
+    for (int i = 0; i < U_SLOTS; ++i) {
+      mbar_init(&u_full[i], 1);
+      mbar_init(&u_empty[i], U_READERS);
     }
     *abort_flag = 0;
     fence_barrier_init();
@@ -171,43 +226,76 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    // -------------------------------------------------- TMA producer
-    // lane 0 loads Q and the K tiles, lane 1 the V tiles, so waiting for a V
-    // buffer (freed by PV) never delays the next K (needed by QK^T).
+    // -------------------------------------------------- TMA producers
+    // lane 0 takes the units from the global counter and loads each unit's
+    // Q tiles (once the previous unit's QK^T are done with them) and its K
+    // tiles; lane 1 loads the V tiles.  Both rings run on across the units
+    // of this CTA.
     if (lane == 0) {
       tma_prefetch_desc(&mQ);
       tma_prefetch_desc(&mKV);
-      mbar_arrive_expect_tx(q_full, nt * TILE_BYTES);
-      for (int t = 0; t < nt; ++t) {
-        tma_load_2d(smem + OFF_Q + t * TILE_BYTES, &mQ, q_full, xq, q0 + t * BQ);
-        tma_load_2d(smem + OFF_Q + t * TILE_BYTES + PANEL, &mQ, q_full, xq + 64, q0 + t * BQ);
-      }
-    }
-    if (lane < 2) {
-      const bool is_k = lane == 0;
-      const int stages = is_k ? K_STAGES : V_STAGES;
-      uint64_t* full = is_k ? k_full : v_full;
-      uint64_t* empty = is_k ? k_empty : v_empty;
-      const int x = is_k ? xk : xv;
-      int issued = 0;
-      for (int j = 0; j < nkv; ++j) {
-        const int st = j % stages, use = j / stages;
-        if (use > 0 && !mbar_wait(&empty[st], (use - 1) & 1, abort_flag, p.err)) break;
-        uint8_t* dst = smem + (is_k ? OFF_K : OFF_V) + st * TILE_BYTES;
-        mbar_arrive_expect_tx(&full[st], TILE_BYTES);
-        tma_load_2d(dst, &mKV, &full[st], x, kv0 + j * BKV);
-        tma_load_2d(dst + PANEL, &mKV, &full[st], x + 64, kv0 + j * BKV);
-        ++issued;
+      int q_issued = 0, issued = 0;
+      bool ok = true;
+      int u = blockIdx.x;
+      unit_slot[0] = u;
+      mbar_arrive(&u_full[0]);
+      for (int i = 0; ok && u >= 0; ++i) {
+        const Unit d = decode_unit(p, u);
+        if (i > 0 && !mbar_wait(q_empty, (i - 1) & 1, abort_flag, p.err)) break;
+        mbar_arrive_expect_tx(q_full, d.nt * TILE_BYTES);
+        for (int t = 0; t < d.nt; ++t) {
+          tma_load_2d(smem + OFF_Q + t * TILE_BYTES, &mQ, q_full, d.xq, d.q0 + t * BQ);
+          tma_load_2d(smem + OFF_Q + t * TILE_BYTES + PANEL, &mQ, q_full, d.xq + 64, d.q0 + t * BQ);
+        }
+        ++q_issued;
+        // publish unit i+1 now, so the V lane can run on into it
+        const int n = i + 1, sl = n % U_SLOTS;
+        if (n >= U_SLOTS && !mbar_wait(&u_empty[sl], (n / U_SLOTS - 1) & 1, abort_flag, p.err)) break;
+        int un = G + atomicAdd(p.work_next, 1);
+        if (un >= count) un = -1;
+        unit_slot[sl] = un;
+        mbar_arrive(&u_full[sl]);
+        for (int j = 0; j < d.nkv; ++j) {
+          const int st = issued % K_STAGES, use = issued / K_STAGES;
+          if (use > 0 && !mbar_wait(&k_empty[st], (use - 1) & 1, abort_flag, p.err)) { ok = false; break; }
+          uint8_t* dst = smem + OFF_K + st * TILE_BYTES;
+          mbar_arrive_expect_tx(&k_full[st], TILE_BYTES);
+          tma_load_2d(dst, &mKV, &k_full[st], d.xk, d.kv0 + j * BKV);
+          tma_load_2d(dst + PANEL, &mKV, &k_full[st], d.xk + 64, d.kv0 + j * BKV);
+          ++issued;
+        }
+        u = un;
       }
       if (*abort_flag) {
-        if (is_k) mbar_wait_drain(q_full, 0, 200000000ull);
-        for (int j = issued > stages ? issued - stages : 0; j < issued; ++j)
-          mbar_wait_drain(&full[j % stages], (j / stages) & 1, 200000000ull);
+        if (q_issued > 0) mbar_wait_drain(q_full, (q_issued - 1) & 1, 200000000ull);
+        for (int j = issued > K_STAGES ? issued - K_STAGES : 0; j < issued; ++j)
+          mbar_wait_drain(&k_full[j % K_STAGES], (j / K_STAGES) & 1, 200000000ull);
+      }
+    } else if (lane == 1) {
+      int issued = 0;
+      bool ok = true;
+      for (int i = 0; ok; ++i) {
+        const int u = read_unit(u_full, u_empty, unit_slot, i, abort_flag, p.err, true);
+        if (u < 0) break;
+        const Unit d = decode_unit(p, u);
+        for (int j = 0; j < d.nkv; ++j) {
+          const int st = issued % V_STAGES, use = issued / V_STAGES;
+          if (use > 0 && !mbar_wait(&v_empty[st], (use - 1) & 1, abort_flag, p.err)) { ok = false; break; }
+          uint8_t* dst = smem + OFF_V + st * TILE_BYTES;
+          mbar_arrive_expect_tx(&v_full[st], TILE_BYTES);
+          tma_load_2d(dst, &mKV, &v_full[st], d.xv, d.kv0 + j * BKV);
+          tma_load_2d(dst + PANEL, &mKV, &v_full[st], d.xv + 64, d.kv0 + j * BKV);
+          ++issued;
+        }
+      }
+      if (*abort_flag) {
+        for (int j = issued > V_STAGES ? issued - V_STAGES : 0; j < issued; ++j)
+          mbar_wait_drain(&v_full[j % V_STAGES], (j / V_STAGES) & 1, 200000000ull);
       }
     }
   } else if (warp == 1 || warp == 2) {
     const int t = warp - 1;
-    if (lane == 0 && t < nt) {
+    if (lane == 0) {
       // ------------------------------------------------ MMA issuer of tile t
       constexpr uint32_t idesc_qk = make_idesc(BQ, BKV, 0, F16);
       constexpr uint32_t idesc_pv = make_idesc(BQ, DH, 1, F16);
@@ -217,45 +305,104 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint64_t dk0 = make_sdesc_sw128(smem_u32(smem + OFF_K), 16, 1024);
       const uint64_t dv0 = make_sdesc_sw128(smem_u32(smem + OFF_V), PANEL, 1024);
       const uint32_t dS = tmem + TM_S + 128 * t, dO = tmem + TM_O + 128 * t;
-      bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
-      for (int j = 0; ok && j <= nkv; ++j) {
-        // everything this round needs, then the turn: round j of tile 1
-        // follows round j of tile 0, which follows round j-1 of tile 1
-        const int jv = j - 1, vs = jv % V_STAGES, ks = j % K_STAGES;
-        if ((j > 0 && (!mbar_wait(&v_full[vs], (jv / V_STAGES) & 1, abort_flag, p.err) ||
-                       !mbar_wait(&p_full[t], jv & 1, abort_flag, p.err))) ||
-            (j < nkv && !mbar_wait(&k_full[ks], (j / K_STAGES) & 1, abort_flag, p.err))) {
-          ok = false;
-          break;
+      // ring positions run on across units: stage = count % 2, phase = count / 2 % 2
+      unsigned kc = 0, vc = 0;       // K / V tiles consumed
+      unsigned pc = 0, tc = 0;       // P tiles consumed, turn waits
+      unsigned oc = 0;               // units of this tile finished
+      bool paired_before = false;    // a unit with both tiles active was seen
+      bool ok = true;
+      // S_t = Q_t K^T for the K tile at ring position kc (both K-major, 128-byte swizzle)
+      auto qk = [&](unsigned c) {
+        const uint64_t dk = dk0 + static_cast<uint64_t>((c & 1u) * (TILE_BYTES >> 4));
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint64_t off = static_cast<uint64_t>(((k >> 2) * PANEL + (k & 3) * 32) >> 4);
+          tc_mma_f16(dS, dq + off, dk + off, idesc_qk, k > 0 ? 1u : 0u);
         }
-        if (nt > 1 && (t == 1 || j > 0) && !mbar_wait(&turn[t], (t == 1 ? j : j - 1) & 1, abort_flag, p.err)) {
-          ok = false;
-          break;
+        tc_commit(&s_full[t]);
+        tc_commit(&k_empty[c & 1u]);
+      };
+      // O_t (+)= P_t V for the V tile at ring position c: A = P from tensor
+      // memory (8 columns per 16 keys), B = V [keys, dims] with dims
+      // contiguous, an MN-major operand whose 64-dim panels are PANEL bytes
+      // apart (LBO) and 8-key groups 1 KB apart (SBO)
+      // (vt: the V tile's index in the unit; tile 0 starts a fresh O_t)
+      auto pv = [&](unsigned c, int vt) {
+        const uint64_t dv = dv0 + static_cast<uint64_t>((c & 1u) * (TILE_BYTES >> 4));
+#pragma unroll
+        for (int k = 0; k < BKV / 16; ++k)
+          tc_mma_f16_tmem_a(dO, dS + 8 * k, dv + static_cast<uint64_t>(k * 128), idesc_pv, (vt > 0 || k > 0) ? 1u : 0u);
+        tc_commit(&v_empty[c & 1u]);
+      };
+      for (int i = 0; ok; ++i) {
+        const int u = read_unit(u_full, u_empty, unit_slot, i, abort_flag, p.err, true);
+        if (u < 0) break;
+        const Unit d = decode_unit(p, u);
+        if (!mbar_wait(q_full, i & 1, abort_flag, p.err)) break;
+        if (t >= d.nt) {
+          // idle this unit: release Q and every K / V stage as they pass
+          mbar_arrive(q_empty);
+          for (int j = 0; j < d.nkv; ++j, ++kc, ++vc) {
+            if (!mbar_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err) ||
+                !mbar_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive(&k_empty[kc & 1u]);
+            mbar_arrive(&v_empty[vc & 1u]);
+          }
+          continue;
+        }
+        const bool pair = d.nt > 1;
+        const int nkv = d.nkv;
+        // rounds: 0 = QK^T of K_0; j = 1 .. nkv-1: PV of V_j-1, then QK^T of
+        // K_j; nkv = PV of V_nkv-1.  Round j of tile 1 follows round j of tile
+        // 0, which follows round j-1 of tile 1 (the turn token); tile 0's
+        // round 0 follows tile 1's last round of the previous paired unit.
+        if (!mbar_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err)) break;
+        if (pair && (t == 1 || paired_before)) {
+          if (!mbar_wait(&turn[t], tc & 1u, abort_flag, p.err)) break;
+          ++tc;
         }
         tc_fence_after();
-        if (j > 0) {
-          // O_t += P_t,j-1 V_j-1: A = P from tensor memory (8 columns per 16
-          // keys); B = V [keys, dims] with dims contiguous, an MN-major
-          // operand whose two 64-dim panels are PANEL bytes apart (LBO) and
-          // 8-key groups 1 KB apart (SBO)
-#pragma unroll
-          for (int k = 0; k < BKV / 16; ++k)
-            tc_mma_f16_tmem_a(dO, dS + 8 * k, dv0 + static_cast<uint64_t>(vs * (TILE_BYTES >> 4) + k * 128), idesc_pv,
-                              (jv > 0 || k > 0) ? 1u : 0u);
-          tc_commit(&v_empty[vs]);
-          if (j == nkv) tc_commit(&o_done[t]);
-        }
-        if (j < nkv) {
-#pragma unroll
-          for (int k = 0; k < DH / 16; ++k) {
-            // A = Q_t, B = K_j, both K-major with 128-byte swizzle
-            const uint64_t off = static_cast<uint64_t>(((k >> 2) * PANEL + (k & 3) * 32) >> 4);
-            tc_mma_f16(dS, dq + off, dk0 + static_cast<uint64_t>(ks * (TILE_BYTES >> 4)) + off, idesc_qk, k > 0 ? 1u : 0u);
+        qk(kc);
+        ++kc;
+        if (nkv == 1) tc_commit(q_empty);
+        if (pair) mbar_arrive(&turn[t ^ 1]);
+        // the first PV overwrites O_t: the previous unit's O_t must be read out
+        if (oc > 0 && !mbar_wait(&o_free[t], (oc - 1) & 1u, abort_flag, p.err)) break;
+        for (int j = 1; j < nkv; ++j) {
+          if (!mbar_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err) ||
+              !mbar_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
+              !mbar_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err) ||
+              (pair && !mbar_wait(&turn[t], tc & 1u, abort_flag, p.err))) {
+            ok = false;
+            break;
           }
-          tc_commit(&s_full[t]);
-          tc_commit(&k_empty[ks]);
+          tc += pair ? 1u : 0u;
+          tc_fence_after();
+          pv(vc, j - 1);
+          qk(kc);
+          ++vc;
+          ++pc;
+          ++kc;
+          if (pair) mbar_arrive(&turn[t ^ 1]);
         }
-        if (nt > 1) mbar_arrive(&turn[t ^ 1]);
+        if (!ok) break;
+        if (nkv > 1) tc_commit(q_empty);
+        if (!mbar_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err) ||
+            !mbar_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
+            (pair && !mbar_wait(&turn[t], tc & 1u, abort_flag, p.err)))
+          break;
+        tc += pair ? 1u : 0u;
+        tc_fence_after();
+        pv(vc, nkv - 1);
+        tc_commit(&o_done[t]);
+        ++vc;
+        ++pc;
+        if (pair) mbar_arrive(&turn[t ^ 1]);
+        if (pair) paired_before = true;
+        ++oc;
       }
     }
   } else if (warp >= 4) {
@@ -267,116 +414,134 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t tS = tmem + lane_off + TM_S + 128 * t;
     const uint32_t tO = tmem + lane_off + TM_O + 128 * t;
     const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
-    float m_ref = -INFINITY;                      // running max, log2 units
-    float l = 0.f;                                // row sum
-    bool ok = t < nt;
-    for (int j = 0; ok && j < nkv; ++j) {
-      // warp-uniform outcomes: the TMEM accesses that follow are warp-collective
-      if (!__all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, abort_flag, p.err))) { ok = false; break; }
-      tc_fence_after();
-      float s[BKV];
-      {
-        uint32_t ra[BKV / 32][32];
-#pragma unroll
-        for (int c = 0; c < BKV / 32; ++c) tmem_ld32(tS + 32 * c, ra[c]);
-        tmem_ld_wait();
-#pragma unroll
-        for (int c = 0; c < BKV / 32; ++c)
-#pragma unroll
-          for (int i = 0; i < 32; ++i) s[32 * c + i] = __uint_as_float(ra[c][i]);
+    int cs = 0, co = 0, cv = 0;                   // S tiles seen, units done (this tile), V tiles before the unit
+    bool ok = true;
+    for (int i = 0; ok; ++i) {
+      const int u = __shfl_sync(0xffffffffu, read_unit(u_full, u_empty, unit_slot, i, abort_flag, p.err, lane == 0), 0);
+      if (u < 0) break;
+      const Unit d = decode_unit(p, u);
+      if (t >= d.nt) {
+        cv += d.nkv;
+        continue;
       }
-      const int valid = kvL - j * BKV;            // keys of this tile, >= 1
-      if (valid < BKV) {
+      float m_ref = -INFINITY;                    // running max, log2 units
+      float l = 0.f;                              // row sum
+      for (int j = 0; ok && j < d.nkv; ++j) {
+        // warp-uniform outcomes: the TMEM accesses that follow are warp-collective
+        if (!__all_sync(0xffffffffu, mbar_wait(&s_full[t], cs & 1, abort_flag, p.err))) { ok = false; break; }
+        ++cs;
+        tc_fence_after();
+        float s[BKV];
+        {
+          uint32_t ra[BKV / 32][32];
 #pragma unroll
-        for (int c = 0; c < BKV; ++c) s[c] = c < valid ? s[c] : -INFINITY;
-      }
-      // row max: eight independent chains, then a tree
-      float mx[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) mx[i] = fmaxf(s[i], s[i + 8]);
-#pragma unroll
-      for (int c = 16; c < BKV; c += 16)
-#pragma unroll
-        for (int i = 0; i < 8; ++i) mx[i] = max3(mx[i], s[c + i], s[c + 8 + i]);
-#pragma unroll
-      for (int w = 4; w >= 1; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) mx[i] = fmaxf(mx[i], mx[i + w]);
-      const float m_new = fmaxf(m_ref, mx[0] * scale_log2);
-      const bool need = (j == 0) || (m_new > m_ref + RESCALE_THRESHOLD);
-      float alpha = 1.f;
-      if (need) {
-        alpha = (j == 0) ? 0.f : ex2(m_ref - m_new);
-        m_ref = m_new;
-      }
-      // P_t,j: keys 32c .. 32c+31 -> 16 packed columns 16c .. 16c+15 of S_t
-      // (the scores were all read above; O_t += P_t,j-1 V_j-1 has completed)
-      const float neg = -m_ref;
-      float rs[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int c = 0; c < BKV / 32; ++c) {
-        uint32_t pk[16];
-        row_probs<F16>(s + 32 * c, scale_log2, neg, rs, pk);
-        tmem_st16(tS + 16 * c, pk);
-      }
-      l = l * alpha + ((rs[0] + rs[1]) + (rs[2] + rs[3]));
-      // rescale O_t in tensor memory if the reference max moved
-      if (j > 0 && __any_sync(0xffffffffu, need)) {
-#pragma unroll 1
-        for (int c = 0; c < DH / 32; ++c) {
-          uint32_t rr[32];
-          tmem_ld32(tO + 32 * c, rr);
+          for (int cc = 0; cc < BKV / 32; ++cc) tmem_ld32(tS + 32 * cc, ra[cc]);
           tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 32; ++i) rr[i] = __float_as_uint(__uint_as_float(rr[i]) * alpha);
-          tmem_st32(tO + 32 * c, rr);
+          for (int cc = 0; cc < BKV / 32; ++cc)
+#pragma unroll
+            for (int e = 0; e < 32; ++e) s[32 * cc + e] = __uint_as_float(ra[cc][e]);
         }
-      }
-      if (valid < BKV) {
-        // last, partial key tile: clear the value rows past kv_len so stale
-        // (possibly non-finite) data cannot meet the zero probabilities (both
-        // groups write the same zeros: each must see them before its PV)
-        const int vst = j % V_STAGES;
-        if (!__all_sync(0xffffffffu, mbar_wait(&v_full[vst], (j / V_STAGES) & 1, abort_flag, p.err))) { ok = false; break; }
-        if (r >= valid) {
+        const int valid = d.kvL - j * BKV;        // keys of this tile, >= 1
+        if (valid < BKV) {
 #pragma unroll
-          for (int pn = 0; pn < 2; ++pn) {
-            uint4* v = reinterpret_cast<uint4*>(smem + OFF_V + vst * TILE_BYTES + pn * PANEL + r * 128);
+          for (int cc = 0; cc < BKV; ++cc) s[cc] = cc < valid ? s[cc] : -INFINITY;
+        }
+        // row max: eight independent chains, then a tree
+        float mx[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = make_uint4(0, 0, 0, 0);
+        for (int e = 0; e < 8; ++e) mx[e] = fmaxf(s[e], s[e + 8]);
+#pragma unroll
+        for (int cc = 16; cc < BKV; cc += 16)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) mx[e] = max3(mx[e], s[cc + e], s[cc + 8 + e]);
+#pragma unroll
+        for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+          for (int e = 0; e < w; ++e) mx[e] = fmaxf(mx[e], mx[e + w]);
+        const float m_new = fmaxf(m_ref, mx[0] * scale_log2);
+        const bool need = (j == 0) || (m_new > m_ref + RESCALE_THRESHOLD);
+        float alpha = 1.f;
+        if (need) {
+          alpha = (j == 0) ? 0.f : ex2(m_ref - m_new);
+          m_ref = m_new;
+        }
+        // P_t,j: keys 32c .. 32c+31 -> 16 packed columns 16c .. 16c+15 of S_t
+        // (the scores were all read above; O_t += P_t,j-1 V_j-1 has completed)
+        const float neg = -m_ref;
+        float rs[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int cc = 0; cc < BKV / 32; ++cc) {
+          uint32_t pk[16];
+          row_probs<F16>(s + 32 * cc, scale_log2, neg, rs, pk);
+          tmem_st16(tS + 16 * cc, pk);
+        }
+        l = l * alpha + ((rs[0] + rs[1]) + (rs[2] + rs[3]));
+        // rescale O_t in tensor memory if the reference max moved
+        if (j > 0 && __any_sync(0xffffffffu, need)) {
+#pragma unroll 1
+          for (int cc = 0; cc < DH / 32; ++cc) {
+            uint32_t rr[32];
+            tmem_ld32(tO + 32 * cc, rr);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
+            tmem_st32(tO + 32 * cc, rr);
           }
         }
-        fence_proxy_async_smem();
+        if (valid < BKV) {
+          // last, partial key tile: clear the value rows past kv_len so stale
+          // (possibly non-finite) data cannot meet the zero probabilities (both
+          // groups write the same zeros: each must see them before its PV)
+          const int vsi = cv + j, vst = vsi % V_STAGES;
+          if (!__all_sync(0xffffffffu, mbar_wait(&v_full[vst], (vsi / V_STAGES) & 1, abort_flag, p.err))) {
+            ok = false;
+            break;
+          }
+          if (r >= valid) {
+#pragma unroll
+            for (int pn = 0; pn < 2; ++pn) {
+              uint4* v = reinterpret_cast<uint4*>(smem + OFF_V + vst * TILE_BYTES + pn * PANEL + r * 128);
+#pragma unroll
+              for (int e = 0; e < 8; ++e) v[e] = make_uint4(0, 0, 0, 0);
+            }
+          }
+          fence_proxy_async_smem();
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[t]);
       }
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[t]);
-    }
-    if (ok && nkv > 0) ok = __all_sync(0xffffffffu, mbar_wait(&o_done[t], 0, abort_flag, p.err));
-    if (ok && nkv > 0) {
+      if (!ok) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&o_done[t], co & 1, abort_flag, p.err))) break;
       tc_fence_after();
       const float inv_l = 1.f / l;
-      const int qrow = (qt0 + t) * BQ + r;        // row inside the segment
-      const bool valid_row = qrow < L;
+      const int qrow = (d.qt0 + t) * BQ + r;      // row inside the segment
+      const bool valid_row = qrow < d.L;
       uint16_t* orow =
-          reinterpret_cast<uint16_t*>(p.out) + static_cast<size_t>(valid_row ? seq0 + qrow : 0) * p.ldo + h * DH;
+          reinterpret_cast<uint16_t*>(p.out) + static_cast<size_t>(valid_row ? d.seq0 + qrow : 0) * p.ldo + d.h * DH;
 #pragma unroll 1
-      for (int c = 0; c < DH / 32; ++c) {
+      for (int cc = 0; cc < DH / 32; ++cc) {
         uint32_t rr[32];
-        tmem_ld32(tO + 32 * c, rr);
+        tmem_ld32(tO + 32 * cc, rr);
         tmem_ld_wait();
         if (valid_row) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + 32 * c);
+          uint4* dst = reinterpret_cast<uint4*>(orow + 32 * cc);
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            dst[i] = make_uint4(pack2(__uint_as_float(rr[8 * i + 0]) * inv_l, __uint_as_float(rr[8 * i + 1]) * inv_l, F16),
-                                pack2(__uint_as_float(rr[8 * i + 2]) * inv_l, __uint_as_float(rr[8 * i + 3]) * inv_l, F16),
-                                pack2(__uint_as_float(rr[8 * i + 4]) * inv_l, __uint_as_float(rr[8 * i + 5]) * inv_l, F16),
-                                pack2(__uint_as_float(rr[8 * i + 6]) * inv_l, __uint_as_float(rr[8 * i + 7]) * inv_l, F16));
+          for (int e = 0; e < 4; ++e) {
+            dst[e] = make_uint4(pack2(__uint_as_float(rr[8 * e + 0]) * inv_l, __uint_as_float(rr[8 * e + 1]) * inv_l, F16),
+                                pack2(__uint_as_float(rr[8 * e + 2]) * inv_l, __uint_as_float(rr[8 * e + 3]) * inv_l, F16),
+                                pack2(__uint_as_float(rr[8 * e + 4]) * inv_l, __uint_as_float(rr[8 * e + 5]) * inv_l, F16),
+                                pack2(__uint_as_float(rr[8 * e + 6]) * inv_l, __uint_as_float(rr[8 * e + 7]) * inv_l, F16));
           }
         }
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&o_free[t]);
+      ++co;
+      cv += d.nkv;
     }
   }
 
@@ -433,7 +598,8 @@ __global__ void attn_schedule_kernel(const int* cu, const int* cu_kv, const int*
       record_error(err, kErrCapacity);
       acc = max_units;
     }
-    *work_count = acc;
+    work_count[0] = acc;
+    work_count[1] = 0;            // next unit handed out by the attention kernel
   }
   __syncthreads();
   for (int i = 0; i < B; ++i) {

@@ -179,6 +179,40 @@ def test_attention_many_heads():
     _attention_case("f16", 4, 128, [200, 90], [200, 90], 1.0, 12)
 
 
+@pytest.mark.parametrize("dt", ["f16", "bf16"])
+def test_attention_many_units_per_cta(dt):
+    # several hundred (segment, head, query-tile pair) units, more than there are
+    # SMs: each persistent CTA takes units in turn, mixing paired and single
+    # query tiles, masked key tails and one-row segments
+    r = _rng(21)
+    lens = [int(x) for x in r.integers(1, 400, 48)]
+    lens[3], lens[7], lens[11] = 1, 256, 257
+    kv = [max(1, L - int(r.integers(0, min(L, 40)))) for L in lens]
+    _attention_case(dt, 8, 128, lens, kv, 1.0, 22)
+
+
+def test_attention_workspace_reused_across_schedules():
+    # the unit counter lives in the schedule workspace: a second call with
+    # another schedule on the same workspace must start from unit 0 again
+    H, dh = 4, 128
+    D = H * dh
+    T_cap = 3000
+    ws_bytes = (H * ((T_cap + 127) // 128 + 64) * 16) + 4096
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=cuda())
+    for seed, lens in ((31, [900, 40, 700, 1, 300]), (32, [129] * 20), (33, [2999])):
+        rng = _rng(seed)
+        cu = np.concatenate([[0], np.cumsum(lens)])
+        T = int(cu[-1])
+        qkv = _store(rng.standard_normal((T_cap, 3 * D)), "f16")
+        out = torch.full((T_cap, D), 3.0, dtype=torch.float16, device=cuda())
+        S.seer_attention(to_dev(qkv, "f16"), out, "f16", i32(cu), None, len(lens), T_cap, H, dh, ws, ws_bytes)
+        ref = np.concatenate([oracle.attention(qkv[a:b, :D], qkv[a:b, D:2 * D], qkv[a:b, 2 * D:3 * D], H)
+                              for a, b in zip(cu[:-1], cu[1:])])
+        got = host(out)
+        check_close(got[:T], ref, "bf16", f"attention reuse lens={lens}")
+        assert (got[T:] == 3.0).all()
+
+
 def test_attention_f32():
     _attention_case("f32", 4, 64, [1, 70, 33, 130], [1, 70, 20, 130], 1.0, 13)
 
