@@ -180,15 +180,17 @@ def test_attention_many_heads():
 
 
 @pytest.mark.parametrize("dt", ["f16", "bf16"])
-def test_attention_many_units_per_cta(dt):
-    # several hundred (segment, head, query-tile pair) units, more than there are
-    # SMs: each persistent CTA takes units in turn, mixing paired and single
-    # query tiles, masked key tails and one-row segments
+@pytest.mark.parametrize("H", [8, 3])
+def test_attention_many_units_per_cta(dt, H):
+    # hundreds of work units, more than there are SMs: each persistent CTA
+    # takes units in turn, mixing paired and single query tiles (odd tile
+    # counts), masked key tails and one-row segments, for an even and an odd
+    # head count
     r = _rng(21)
     lens = [int(x) for x in r.integers(1, 400, 48)]
     lens[3], lens[7], lens[11] = 1, 256, 257
     kv = [max(1, L - int(r.integers(0, min(L, 40)))) for L in lens]
-    _attention_case(dt, 8, 128, lens, kv, 1.0, 22)
+    _attention_case(dt, H, 128, lens, kv, 1.0, 22)
 
 
 def test_attention_workspace_reused_across_schedules():
