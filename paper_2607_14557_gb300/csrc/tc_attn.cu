@@ -58,6 +58,7 @@ constexpr int TILE_BYTES = 128 * DH * 2;    // 32 KB: 128 rows x 128 16-bit valu
 constexpr int PANEL = 16384;
 constexpr int K_STAGES = 2;                 // 3 measured 1% slower
 constexpr int V_STAGES = 2;
+static_assert(K_STAGES == 2 && V_STAGES == 2, "the MMA issuer takes ring stage = count & 1, phase = count >> 1 & 1");
 constexpr int OFF_Q = 0;                                   // Q tiles 0, 1
 constexpr int OFF_K = NT * TILE_BYTES;
 constexpr int OFF_V = OFF_K + K_STAGES * TILE_BYTES;
