@@ -277,7 +277,10 @@ seer_status seer_convert(const void* src, seer_dtype src_dt, void* dst, seer_dty
 
 /* o[T, H*dh]: per segment b and head h, softmax(q k^T / sqrt(dh)) v over the
  * segment's first kv_len[b] keys (Eqs. 6-7, no causal mask).  qkv [T, 3*H*dh]
- * holds q | k | v.  ws as for seer_layer_forward (only the scheduling part). */
+ * holds q | k | v.  ws as for seer_layer_forward (only the scheduling part:
+ * the work units, their count and the counter from which the attention
+ * kernel's persistent CTAs take units; all rewritten by every call, so calls
+ * that share a workspace must not overlap on the GPU). */
 seer_status seer_attention(const void* qkv, void* o, seer_dtype dt, const int32_t* cu_seqlens,
                            const int32_t* kv_len, int B, int T_capacity, int n_heads, int head_dim,
                            void* ws, size_t ws_bytes, void* stream);
