@@ -6,7 +6,14 @@ step-0 boundary detection (SwiGLU GEMM + fused sparsity count + SNR scan),
 routing + device-resident compaction, and one truncated denoising layer
 (RMSNorm, QKV, varlen bidirectional attention, O projection, SwiGLU MLP).
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 2] [--impl ours|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload suite|0..4] [--impl ours|reference]
+
+The default run (``--workload suite``) leads with the video-shaped layer
+(workload 4: batch 4, 11.8k-row visual prefixes, window 2048), the largest
+single-layer configuration, and carries the ragged batch-16 layer (workload 2)
+and the 32-layer x 64-step stack (workload 3) as sub-records of the same line,
+each with its own timing, roofline, oracle baseline, end-to-end figure and
+clock record.
 
 ``value``  valid tokens per second of the device-resident step (inputs in HBM);
 ``e2e``    the same metric with the host->device copy of the step's input and
@@ -38,6 +45,19 @@ PRECISION = "bf16 layer inputs/outputs, f16 tensor-core operands and intermediat
 METRIC = "truncated denoise-layer tokens/s & TFLOP/s vs BF16 peak; speedup over padded"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 KERNELS_PER_STEP = 11   # detect GEMM, scan, pack, norm, QKV, attn schedule, attn, O proj, norm, gate/up, down
+SUITE = (4, 2, 3)       # headline first: the video layer, then the ragged batch-16 layer and the 32-layer stack
+TENSOR_PHASES = ("detect_gemm", "qkv", "attention", "o_proj", "gate_up", "down")
+KERNEL_OF_PHASE = {
+    "detect_gemm": "tc_gemm_kernel<Count> (step-0 detector, counts only)",
+    "qkv": "tc_gemm_kernel<Store> (QKV projection)",
+    "attention": "tc_attn_kernel (varlen bidirectional attention)",
+    "o_proj": "tc_gemm_kernel<Residual> (O projection + residual)",
+    "gate_up": "tc_gemm_kernel<Swiglu> (gate/up + SwiGLU)",
+    "down": "tc_gemm_kernel<Residual> (down projection + residual)",
+}
+# kept rows above which the oracle's layer time is scaled from a sample of
+# query rows instead of measured on every row
+ORACLE_FULL_ROWS = 4096
 
 
 def parse():
@@ -45,7 +65,7 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", type=int, default=2, choices=[0, 1, 2, 3, 4])
+    ap.add_argument("--workload", default="suite", choices=["suite", "0", "1", "2", "3", "4"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -79,17 +99,18 @@ def code_digest(paths) -> str:
     return h.hexdigest()
 
 
-def measured_traffic(workload: int, kernel: str):
-    """DRAM bytes per launch of `kernel` from the committed ncu capture of this
-    workload, or None when the kernel code changed since that capture."""
+def measured_traffic(workload: int, phase: str):
+    """DRAM bytes per launch of the kernel of `phase` from the committed ncu
+    capture of this workload, or None when the kernel code changed since that
+    capture."""
     path = os.path.join(ROOT, "profiles", f"traffic_workload{workload}.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         doc = json.load(f)
-    if code_digest(doc["sources"]) != doc.get("sources_code_sha1") or kernel not in doc["kernels"]:
+    if code_digest(doc["sources"]) != doc.get("sources_code_sha1") or phase not in doc["kernels"]:
         return None
-    return doc["kernels"][kernel]["traffic_bytes"]
+    return doc["kernels"][phase]["traffic_bytes"]
 
 
 def graph_capacity(total: int) -> int:
@@ -170,7 +191,18 @@ _ORACLE_INPUTS = {}
 
 def oracle_sample(wl):
     """Time the CPU oracle on one sequence of the workload (the shortest one):
-    its detection window, boundary scan, and one truncated layer."""
+    detection over its whole window, the boundary scan, and one truncated layer
+    over its kept rows.
+
+    Where the kept rows exceed ORACLE_FULL_ROWS (the video workload: ~12k rows,
+    about a minute of fp64 work), the layer runs on a sample of query rows (keys
+    and values still from every kept row) and its time is scaled to the whole
+    layer by the algorithmic FLOP count: K/V projections 4*keep*d^2 always,
+    plus per query row 4*d^2 (Q, O) + 6*d*F (MLP) + 4*d*keep (attention).  The
+    oracle is BLAS-bound, so its time follows the FLOPs.
+
+    Returns ``(kept_rows, seconds, description)``, seconds being the detection
+    time plus the (possibly extrapolated) layer time."""
     import oracle
     if wl.index not in _ORACLE_INPUTS:
         lens = synth.lengths(wl)
@@ -184,10 +216,55 @@ def oracle_sample(wl):
     _, L = oracle.snr_boundary(counts, wl.d_ff)
     keep = int(lens.ctx[b] + L)
     seg = x[cu_full[b]:cu_full[b] + keep]
-    oracle.layer_forward_segment(seg, w, wl.n_heads)
-    dt = time.perf_counter() - t0
-    return keep, dt, f"sequence {b} ({keep} kept rows of {int(lens.full[b])}): detection over its {wl.window}-token " \
-                      f"window + one truncated layer, fp64 numpy"
+    t_detect = time.perf_counter() - t0
+    if keep <= ORACLE_FULL_ROWS:
+        t1 = time.perf_counter()
+        oracle.layer_forward_segment(seg, w, wl.n_heads)
+        t_layer = time.perf_counter() - t1
+        how = "one truncated layer"
+    else:
+        n = 512
+        q_rows = np.sort(np.random.default_rng(0).choice(keep, size=n, replace=False))
+        t1 = time.perf_counter()
+        oracle.layer_forward_rows(seg, w, wl.n_heads, q_rows)
+        t_n = time.perf_counter() - t1
+        d, F = wl.d, wl.d_ff
+        per_row = 4.0 * d * d + 6.0 * d * F + 4.0 * d * keep
+        t_layer = t_n * (4.0 * keep * d * d + keep * per_row) / (4.0 * keep * d * d + n * per_row)
+        how = (f"one truncated layer, scaled by FLOPs from {n} sampled query rows (keys/values from all {keep} "
+               f"rows; {t_n:.2f} s measured)")
+    dt = t_detect + t_layer
+    return keep, dt, (f"sequence {b} ({keep} kept rows of {int(lens.full[b])}): detection over its {wl.window}-token "
+                      f"window + {how}, fp64 numpy")
+
+
+def layer_config(wl, world, args, L, groups, pad_rows, capacity, T_full, T_valid, T_exec) -> dict:
+    """``config`` of a layer workload (the same dict in both arms)."""
+    d, F = wl.d, wl.d_ff
+    es = 2 if wl.dtype == "bf16" else 4
+    return {"workload": f"{wl.name} (workload {wl.index}): batch {wl.batch}, window {wl.window}, "
+                        f"d {d}, heads {wl.n_heads}x{wl.head_dim}, F {F}",
+            "batch": wl.batch, "window": wl.window, "tokens_full": T_full, "tokens_valid": T_valid,
+            "tokens_executed": T_exec, "L_star": [int(v) for v in L],
+            "l2": "inputs larger than L2 (x_full %.0f MB, weights %.0f MB)" % (T_full * d * es / 1e6,
+                                                                              (4 * d * d + 3 * d * F) * 2 / 1e6),
+            "route": {"groups": groups, "pad_rows": int(pad_rows), "capacity": int(capacity)},
+            "parallelism": f"replicas x{world}", "launch_overlap": args.launch_overlap}
+
+
+def stack_config(wl, args, L, groups, capacity, T_full, T_valid, T_exec) -> dict:
+    d, F = wl.d, wl.d_ff
+    return {"workload": f"{wl.name} (workload 3): {wl.n_layers} layers x {wl.steps} denoising steps, batch "
+                        f"{wl.batch}, window {wl.window}, d {d}, F {F}; tokens counted once per layer and step",
+            "tokens_full": T_full, "tokens_valid": T_valid, "tokens_executed": T_exec, "L_star": [int(v) for v in L],
+            "route": {"groups": groups, "capacity": int(capacity)},
+            "l2": "inputs larger than L2 (weights %.1f GB)" % (wl.n_layers * (4 * d * d + 3 * d * F) * 2 / 1e9),
+            "launch_overlap": args.launch_overlap}
+
+
+def suite_note() -> str:
+    return ("headline: workload 4 (the largest single-layer configuration); sub_records: workload 2 (ragged "
+            "batch-16 layer) and workload 3 (32-layer x 64-step stack)")
 
 
 def reference_config(wl, world, args) -> dict:
@@ -200,30 +277,17 @@ def reference_config(wl, world, args) -> dict:
     tau = 0.2
     seg, kv, cu = oracle.segment_layout(lens.ctx, L, wl.window, tau)
     T_full, T_valid, T_exec = int(lens.full.sum()), int(kv.sum()), int(cu[-1])
+    route = oracle.route(L, wl.window, tau)
     groups = [{"bucket": g["bucket"], "members": len(g["members"]), "path": g["path"],
-               "rho": int(np.floor(g["rho"] * 1e6)) / 1e6} for g in oracle.route(L, wl.window, tau)]
+               "rho": int(np.floor(g["rho"] * 1e6)) / 1e6} for g in route]
     pad = int(sum(g["bucket"] * len(g["members"]) - int(L[g["members"]].sum())
-                  for g in oracle.route(L, wl.window, tau) if g["path"] == oracle.PATH_STATIC))
-    d, F = wl.d, wl.d_ff
+                  for g in route if g["path"] == oracle.PATH_STATIC))
     if wl.index == 3:
-        return {"workload": f"{wl.name} (workload 3): {wl.n_layers} layers x {wl.steps} denoising steps, batch "
-                            f"{wl.batch}, window {wl.window}, d {d}, F {F}; tokens counted once per layer and step",
-                "tokens_full": T_full, "tokens_valid": T_valid, "tokens_executed": T_exec, "L_star": L.tolist(),
-                "route": {"groups": groups, "capacity": graph_capacity(T_exec)},
-                "l2": "inputs larger than L2 (weights %.1f GB)" % (wl.n_layers * (4 * d * d + 3 * d * F) * 2 / 1e9),
-                "launch_overlap": args.launch_overlap}
-    es = 2 if wl.dtype == "bf16" else 4
-    return {"workload": f"{wl.name} (workload {wl.index}): batch {wl.batch}, window {wl.window}, "
-                        f"d {d}, heads {wl.n_heads}x{wl.head_dim}, F {F}",
-            "batch": wl.batch, "window": wl.window, "tokens_full": T_full, "tokens_valid": T_valid,
-            "tokens_executed": T_exec, "L_star": L.tolist(),
-            "l2": "inputs larger than L2 (x_full %.0f MB, weights %.0f MB)" % (T_full * d * es / 1e6,
-                                                                              (4 * d * d + 3 * d * F) * 2 / 1e6),
-            "route": {"groups": groups, "pad_rows": pad, "capacity": graph_capacity(T_exec)},
-            "parallelism": f"replicas x{world}", "launch_overlap": args.launch_overlap}
+        return stack_config(wl, args, L, groups, graph_capacity(T_exec), T_full, T_valid, T_exec)
+    return layer_config(wl, world, args, L, groups, pad, graph_capacity(T_exec), T_full, T_valid, T_exec)
 
 
-def run_reference(args, wl, rank, world):
+def run_reference(args, wl, rank, world, suite):
     if rank != 0:
         return
     cores = len(os.sched_getaffinity(0))
@@ -236,32 +300,66 @@ def run_reference(args, wl, rank, world):
         toks += k
         secs += dt
     v = toks / secs
+    cfg = reference_config(wl, world, args)
+    if suite:
+        cfg["suite"] = suite_note()
     line = {"metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": reference_config(wl, world, args),
+            "config": cfg,
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
+def cpu_baseline(wl, unit="tokens/s"):
+    k, dt, sample = oracle_sample(wl)
+    return {"value": k / dt, "unit": unit, "cores": len(os.sched_getaffinity(0)), "kind": "oracle",
+            "sample": sample, "seconds": dt}
+
+
+# ----------------------------------------------------------------- environment of our arm
+class Env:
+    def __init__(self):
+        import torch
+        import torch.distributed as dist
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        torch.cuda.set_device(self.local)
+        self.dev = torch.device("cuda", self.local)
+        if self.world > 1:
+            dist.init_process_group("nccl", device_id=self.dev)
+        from paper_2607_14557_gb300 import replicas as R
+        self.R = R
+
+    def barrier(self):
+        self.R.barrier(self.dev)
+
+    def max_over_ranks(self, v):
+        return self.R.max_over_ranks(v, self.dev)
+
+    def sum_over_ranks(self, v):
+        return self.R.sum_over_ranks(v, self.dev)
+
+    def close(self):
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
 # ----------------------------------------------------------------- stack (workload 3)
-def run_stack(args, wl, world, rank, local):
+def run_stack(args, wl, env, with_cpu):
     """32-layer stack, 64 denoising steps: step 0 over the full windows (with the
     fused count hook at the detection layer), detection + route/pack, then 63
     truncated steps replayed from a CUDA graph; against 64 untruncated steps
-    replayed from their own graph."""
+    replayed from their own graph.  Returns the JSON record."""
     import torch
 
     from paper_2607_14557_gb300 import driver as D
     from paper_2607_14557_gb300 import seer as S
 
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=dev)
-    from paper_2607_14557_gb300 import replicas as R
+    dev, world, R = env.dev, env.world, env.R
     detect_layer = 3
     lens = synth.lengths(wl)
     x_np, cu_full_np, resp_np = synth.hidden_full(wl, lens)
@@ -297,8 +395,8 @@ def run_stack(args, wl, world, rank, local):
     d, F, nl = wl.d, wl.d_ff, wl.n_layers
 
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
-    R.barrier(dev)
-    with ClockSampler(local) as clk:
+    env.barrier()
+    with ClockSampler(env.local) as clk:
         ev[0].record(stream)
         stack.step0(x_full, cu_full, resp, ctx, stream)
         ev[1].record(stream)
@@ -326,7 +424,7 @@ def run_stack(args, wl, world, rank, local):
     torch.cuda.synchronize()
     assert S.seer_check_device() == 0
     evc = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-    with ClockSampler(local) as clk_c:
+    with ClockSampler(env.local) as clk_c:
         evc[0].record(stream)
         stack.step0(x_full, cu_full, resp, ctx, stream)
         evc[1].record(stream)
@@ -365,7 +463,8 @@ def run_stack(args, wl, world, rank, local):
         torch.cuda.synchronize()
         ms_e2e = max(a_e.elapsed_time(b_e), (time.perf_counter() - t_e) * 1e3)
         tok_e = (T_full + (n_steps - 1) * T_valid) * wl.n_layers
-        e2e = {"value": tok_e / (ms_e2e * 1e-3), "unit": "tokens/s", "ms_per_generation": ms_e2e,
+        e2e = {"value": env.sum_over_ranks(tok_e) / (env.max_over_ranks(ms_e2e) * 1e-3), "unit": "tokens/s",
+               "ms_per_generation": ms_e2e,
                "h2d_bytes_per_step": x_host.numel() * x_host.element_size() / n_steps,
                "d2h_bytes_per_step": (r_e["total"] * wl.d * 2 + wl.batch * 4) / n_steps,
                "note": "one generation (64 steps): the input uploaded once, the last step's rows downloaded once"}
@@ -384,23 +483,20 @@ def run_stack(args, wl, world, rank, local):
     tok_layers = (T_full + (n_steps - 1) * T_valid) * nl
     # replicas: every rank runs its own batch; the job's rate is all ranks'
     # token-layers over the slowest rank's time
-    value = R.sum_over_ranks(tok_layers, dev) / (R.max_over_ranks(ms_seer, dev) * 1e-3)
+    value = env.sum_over_ranks(tok_layers) / (env.max_over_ranks(ms_seer) * 1e-3)
     pk, src = peaks()
     tflops_rest = fl_trunc * (n_steps - 1) / (ms_rest * 1e-3) / 1e12
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": n_steps,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_seer / n_steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f16", "precision": PRECISION, "data": "synthetic",
-        "config": {"workload": f"{wl.name} (workload 3): {nl} layers x {n_steps} denoising steps, batch {wl.batch}, "
-                               f"window {wl.window}, d {d}, F {F}; tokens counted once per layer and step",
-                   "tokens_full": T_full, "tokens_valid": T_valid, "tokens_executed": T_exec, "L_star": L.tolist(),
-                   "route": {"groups": r["groups"], "capacity": r["capacity"]},
-                   "l2": "inputs larger than L2 (weights %.1f GB)" % (nl * (4 * d * d + 3 * d * F) * 2 / 1e9),
-                   "weights_setup_s": t_weights, "launch_overlap": args.launch_overlap},
+        "config": dict(stack_config(wl, args, L, r["groups"], r["capacity"], T_full, T_valid, T_exec),
+                       weights_setup_s=t_weights),
         "stack": {"ms_step0_full": ms0, "ms_steps_1_to_%d" % (n_steps - 1): ms_rest, "ms_padded_%d_steps" % n_steps: ms_pad,
                   "speedup_vs_padded": ms_pad / ms_seer,
                   "ideal_ratio": fl_full * n_steps / (fl_full + fl_valid * (n_steps - 1)),
                   "tflops_truncated_steps": tflops_rest, "frac_of_burst_peak": tflops_rest / pk["bf16_tflops"],
+                  "frac_of_sustained_peak": tflops_rest / pk["bf16_tflops_sustained"],
                   "tflops_padded": fl_full * n_steps / (ms_pad * 1e-3) / 1e12,
                   "truncated_tokens_per_s": T_valid * nl * (n_steps - 1) / (ms_rest * 1e-3)},
         "step0_truncated_after_detection": {
@@ -425,53 +521,24 @@ def run_stack(args, wl, world, rank, local):
                         + (nl * 8 + 3) + nl * 13 + (n_steps - 2) * (2 + nl * 9), "clocks": clk.summary(),
         "peak_source": src,
     }
-    if world == 1 and rank == 0 and not args.no_cpu_baseline:
-        k, dt, sample = oracle_sample(wl)
-        line["cpu_baseline"] = {"value": k / dt, "unit": "tokens/s (token-layers: one layer pass)",
-                                "cores": len(os.sched_getaffinity(0)), "kind": "oracle", "sample": sample,
-                                "seconds": dt}
-    if rank == 0:
-        print(json.dumps(line), flush=True)
+    if with_cpu:
+        line["cpu_baseline"] = cpu_baseline(wl, "tokens/s (token-layers: one layer pass)")
+    del stack, layers, x_full, g, g_trunc, g_pad, g_cached
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return line
 
 
-# ----------------------------------------------------------------- our arm
-def main():
-    args = parse()
-    wl = synth.workload(args.workload)
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    if args.impl == "reference":
-        run_reference(args, wl, rank, world)
-        return
-    from paper_2607_14557_gb300 import seer as S_
-
-    S_.seer_set_launch_overlap(args.launch_overlap == "on")
-    if args.workload == 3:
-        run_stack(args, wl, world, rank, local)
-        return
-
+# ----------------------------------------------------------------- a single-layer workload
+def run_layer(args, wl, env, with_cpu):
+    """Detect + route/pack + one truncated layer per step (workloads 0, 1, 2, 4).
+    Returns the JSON record."""
     import torch
-    import torch.distributed as dist
 
     from paper_2607_14557_gb300 import driver as D
     from paper_2607_14557_gb300 import seer as S
 
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=dev)
-
-    from paper_2607_14557_gb300 import replicas as R
-
-    def barrier():
-        R.barrier(dev)
-
-    def max_over_ranks(v):
-        return R.max_over_ranks(v, dev)
-
-    def sum_over_ranks(v):
-        return R.sum_over_ranks(v, dev)
+    dev, world = env.dev, env.world
 
     # ---- synthetic inputs, resident in HBM before timing
     lens = synth.lengths(wl)
@@ -479,6 +546,7 @@ def main():
     w_np = synth.layer_weights(wl, 0)
     tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
     x_host = torch.from_numpy(x_np).to(tdt).pin_memory()
+    del x_np
     x_full = x_host.to(dev)
     i32 = lambda a: torch.as_tensor(np.asarray(a, dtype=np.int32)).to(dev)
     cu_full, resp, ctx = i32(cu_full_np), i32(resp_np), i32(lens.ctx)
@@ -508,25 +576,12 @@ def main():
     flops_exec = layer_flops(seg, kv, d, F)
     flops_valid = layer_flops(kv, kv, d, F)
     flops_pad = layer_flops(lens.full, lens.full, d, F)
+    flops_of = {"qkv": 6.0 * T_exec * d * d, "o_proj": 2.0 * T_exec * d * d, "gate_up": 4.0 * T_exec * d * F,
+                "down": 2.0 * T_exec * d * F, "attention": 4.0 * d * float(np.sum(seg * kv)),
+                "detect_gemm": 4.0 * wl.batch * wl.window * d * F}
 
-    # ---- timed region: K whole steps (device-resident inputs > L2); CUDA events
-    # only around the roofline kernel (gate/up), so launch overlap elsewhere is kept
-    barrier()
-    S.seer_profile_reset()
-    S.seer_profile_select(["gate_up"])
-    S.seer_profile_enable(True)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local) as clk:
-        e0.record(stream)
-        for _ in range(args.steps):
-            step()
-        e1.record(stream)
-        barrier()
-    S.seer_profile_enable(False)
-    ms_step = e0.elapsed_time(e1) / args.steps
-    gate_up_timed = S.seer_profile_read()["gate_up"]
-
-    # ---- per-kernel breakdown: the same K steps again, every phase bracketed by events
+    # ---- per-kernel breakdown (untimed for the headline): the same steps with
+    # events around every phase; it also names the dominant kernel
     S.seer_profile_reset()
     S.seer_profile_select(None)
     S.seer_profile_enable(True)
@@ -535,9 +590,28 @@ def main():
     torch.cuda.synchronize()
     S.seer_profile_enable(False)
     phases = S.seer_profile_read()
-    phases["gate_up"] = gate_up_timed
-    ms_step_max = max_over_ranks(ms_step)
-    tokens_all = sum_over_ranks(T_valid)
+    tensor_ms = {p: phases[p][0] for p in TENSOR_PHASES if phases.get(p, (0, 0))[1]}
+    dominant = max(tensor_ms, key=tensor_ms.get) if wl.dtype == "bf16" else "gate_up"
+
+    # ---- timed region: K whole steps (device-resident inputs > L2); CUDA events
+    # only around the dominant kernel, so launch overlap elsewhere is kept
+    env.barrier()
+    S.seer_profile_reset()
+    S.seer_profile_select([dominant])
+    S.seer_profile_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(env.local) as clk:
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        env.barrier()
+    S.seer_profile_enable(False)
+    ms_step = e0.elapsed_time(e1) / args.steps
+    dominant_timed = S.seer_profile_read()[dominant]
+    phases[dominant] = dominant_timed
+    ms_step_max = env.max_over_ranks(ms_step)
+    tokens_all = env.sum_over_ranks(T_valid)
     value = tokens_all / (ms_step_max * 1e-3)
 
     # ---- layer-only timings: truncated vs untruncated (padded) window
@@ -547,17 +621,17 @@ def main():
         # each comparison starts from the same thermal state: a second idle, then
         # two untimed calls (the truncated, padded and naive layers run back to
         # back otherwise, and the later ones would meet a power-capped clock)
-        barrier()
+        env.barrier()
         time.sleep(1.0)
         for _ in range(2):
             fn()
-        barrier()
+        env.barrier()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         for _ in range(n):
             fn()
         b.record(stream)
-        barrier()
+        env.barrier()
         return a.elapsed_time(b) / n
 
     ms_layer = timed(lambda: path.layer(W, stream=stream), args.steps)
@@ -570,6 +644,12 @@ def main():
     seg_nv = np.diff(cu_nv.cpu().numpy())
     flops_naive = layer_flops(seg_nv, kv_nv.cpu().numpy(), d, F)
     del x_nv, y_nv
+    # the router's padding priced: the same batch with the static path switched
+    # off (every segment keeps exactly ctx + L* rows), layer against layer
+    x_vo, cu_vo, kv_vo, T_vo = path.varlen_only_inputs(x_full, cu_full, ctx, stream)
+    ms_varlen = timed(lambda: path.layer(W, x=x_vo, cu=cu_vo, kv=kv_vo, T_cap=T_vo, stream=stream), args.steps)
+    T_vo_exec = int(cu_vo[-1].item())
+    del x_vo
 
     # ---- end to end through the API with host buffers
     e2e = None
@@ -581,16 +661,16 @@ def main():
         # downloads its packed output and L*; copies overlap neighbouring steps' compute
         copy_stream = torch.cuda.Stream(dev)
         path.run_from_host(x_host, cu_full, resp, ctx, W, y_host, L_host, 2, stream, copy_stream)
-        barrier()
+        env.barrier()
         t0 = time.perf_counter()
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
         r = path.run_from_host(x_host, cu_full, resp, ctx, W, y_host, L_host, args.steps, stream, copy_stream)
         b.record(stream)
-        barrier()
+        env.barrier()
         # the call returns after its last copy: the host clock bounds the whole region
-        ms_e2e = max_over_ranks(max(a.elapsed_time(b), (time.perf_counter() - t0) * 1e3) / args.steps)
+        ms_e2e = env.max_over_ranks(max(a.elapsed_time(b), (time.perf_counter() - t0) * 1e3) / args.steps)
         h2d = x_host.numel() * x_host.element_size()
         d2h = r["total"] * d * x_host.element_size() + wl.batch * 4
         e2e = {"value": tokens_all / (ms_e2e * 1e-3), "unit": "tokens/s", "ms_per_step": ms_e2e,
@@ -599,35 +679,44 @@ def main():
 
     assert S.seer_check_device() == 0
 
-    # ---- roofline of the dominant kernel (gate/up GEMM, tensor bound)
+    # ---- roofline of the dominant kernel
     pk, src = peaks()
     kernels = {}
     for name, (ms, n) in phases.items():
         if n:
             kernels[name] = {"ms_per_launch": ms / n, "launches": n}
-    flops_of = {"qkv": 6.0 * T_exec * d * d, "o_proj": 2.0 * T_exec * d * d, "gate_up": 4.0 * T_exec * d * F,
-                "down": 2.0 * T_exec * d * F, "attention": 4.0 * d * float(np.sum(seg * kv)),
-                "detect_gemm": 4.0 * wl.batch * wl.window * d * F}
     for name, fl in flops_of.items():
         if name in kernels:
             kernels[name]["tflops"] = fl / (kernels[name]["ms_per_launch"] * 1e-3) / 1e12
+            kernels[name]["frac_of_burst_peak"] = kernels[name]["tflops"] / pk["bf16_tflops"]
     es = 2 if wl.dtype == "bf16" else 4
     bytes_of = {"pack": 2.0 * T_exec * d * es, "norm1": T_exec * d * (es + 2), "norm2": T_exec * d * 4}
     for name, by in bytes_of.items():
         if name in kernels:
             kernels[name]["gbs"] = by / (kernels[name]["ms_per_launch"] * 1e-3) / 1e9
-    gu = kernels.get("gate_up", {})
-    achieved = gu.get("tflops")
-    # the timed region is ~0.1 s at full clocks: the burst figure is the denominator
-    # (the sustained one, a seconds-long loop under the power cap, is reported beside it)
+    dk = kernels.get(dominant, {})
+    achieved = dk.get("tflops")
+    # algorithmic bytes per launch of each tensor kernel (operands read once,
+    # outputs written once; intermediates are f16)
+    alg_bytes = {"gate_up": 2.0 * T_exec * d + 2 * 2 * F * d + 2.0 * T_exec * F,
+                 "down": 2.0 * T_exec * F + 2.0 * F * d + 2 * 2.0 * T_exec * d,
+                 "qkv": 2.0 * T_exec * d + 2.0 * 3 * d * d + 2.0 * T_exec * 3 * d,
+                 "o_proj": 2.0 * T_exec * d + 2.0 * d * d + 2 * 2.0 * T_exec * d,
+                 "attention": 2.0 * T_exec * 3 * d + 2.0 * T_exec * d,
+                 "detect_gemm": 2.0 * wl.batch * wl.window * d + 2 * 2 * F * d}
+    # the timed region is well under a second at full clocks: the burst figure is
+    # the denominator (the sustained one, a seconds-long loop under the power
+    # cap, is reported beside it)
     peak = pk["bf16_tflops"]
-    roofline = {"kernel": "tc_gemm_kernel<Swiglu> (gate/up + SwiGLU)", "bound": "tensor", "achieved": achieved,
-                "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak if achieved else None,
+    roofline = {"kernel": KERNEL_OF_PHASE.get(dominant, dominant), "phase": dominant, "bound": "tensor",
+                "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak if achieved else None,
                 "frac_of_sustained": achieved / pk["bf16_tflops_sustained"] if achieved else None,
-                "traffic": measured_traffic(wl.index, "gate_up"),
-                "algorithmic_bytes": float(2 * T_exec * d + 2 * 2 * F * d + 2 * T_exec * F),
+                "traffic": measured_traffic(wl.index, dominant),
+                "algorithmic_bytes": float(alg_bytes[dominant]),
                 "peak_source": f"{src} bf16 dense, burst (f16 operands run at the bf16 rate)",
-                "flops_per_launch": flops_of["gate_up"]}
+                "flops_per_launch": flops_of[dominant],
+                "why_this_kernel": "the tensor-core kernel with the largest share of the step's time "
+                                   "(per-phase CUDA events)"}
 
     clocks = clk.summary()
     line = {
@@ -636,14 +725,8 @@ def main():
         "vs_baseline": None, "dtype": "f16" if wl.dtype == "bf16" else "f32",
         "precision": PRECISION if wl.dtype == "bf16" else "fp32 storage and arithmetic (CUDA cores)",
         "data": "synthetic",
-        "config": {"workload": f"{wl.name} (workload {wl.index}): batch {wl.batch}, window {wl.window}, "
-                               f"d {wl.d}, heads {wl.n_heads}x{wl.head_dim}, F {wl.d_ff}",
-                   "batch": wl.batch, "window": wl.window, "tokens_full": T_full, "tokens_valid": T_valid,
-                   "tokens_executed": T_exec, "L_star": L.tolist(),
-                   "l2": "inputs larger than L2 (x_full %.0f MB, weights %.0f MB)" % (
-                       T_full * d * es / 1e6, (4 * d * d + 3 * d * F) * 2 / 1e6),
-                   "route": {"groups": route["groups"], "pad_rows": route["pad_rows"], "capacity": route["capacity"]},
-                   "parallelism": f"replicas x{world}", "launch_overlap": args.launch_overlap},
+        "config": layer_config(wl, world, args, L, route["groups"], route["pad_rows"], route["capacity"], T_full,
+                               T_valid, T_exec),
         "layer": {"ms_truncated": ms_layer, "ms_padded": ms_pad, "tflops": flops_exec / (ms_layer * 1e-3) / 1e12,
                   "frac_of_burst_peak": flops_exec / (ms_layer * 1e-3) / 1e12 / pk["bf16_tflops"],
                   "frac_of_sustained_peak": flops_exec / (ms_layer * 1e-3) / 1e12 / pk["bf16_tflops_sustained"],
@@ -651,21 +734,62 @@ def main():
                   "flops_executed": flops_exec, "flops_valid": flops_valid, "flops_padded": flops_pad},
         "naive_pad": {"ms": ms_naive, "tokens_executed": int(T_nv), "flops_executed": flops_naive,
                       "speedup_truncated_vs_naive": ms_naive / ms_layer, "ideal_ratio": flops_naive / flops_valid},
+        "route_cost": {"tau_pad": 0.2, "pad_rows": int(route["pad_rows"]), "tokens_executed": T_exec,
+                       "ms_layer": ms_layer, "ms_layer_varlen_only": ms_varlen,
+                       "tokens_executed_varlen_only": T_vo_exec, "ms_cost_of_pad_rows": ms_layer - ms_varlen,
+                       "note": "static-path groups pad their responses to the bucket (rows computed as queries, "
+                               "masked as keys); varlen-only keeps ctx + L* rows in every segment"},
         "speedup_step_vs_padded_layer": ms_pad / ms_step,
         "kernels": kernels,
-        "kernel_timing": "gate_up: CUDA events around that kernel alone inside the timed region; the other "
-                         "kernels: a second pass of the same steps with events around every phase",
+        "kernel_timing": f"{dominant}: CUDA events around that kernel alone inside the timed region; the other "
+                         "kernels: a separate pass of the same steps with events around every phase",
         "roofline": roofline, "gpu_launches": KERNELS_PER_STEP * args.steps,
         "e2e": e2e, "clocks": clocks,
     }
-    if world == 1 and rank == 0 and not args.no_cpu_baseline:
-        k, dt, sample = oracle_sample(wl)
-        line["cpu_baseline"] = {"value": k / dt, "unit": "tokens/s", "cores": len(os.sched_getaffinity(0)),
-                                "kind": "oracle", "sample": sample, "seconds": dt}
-    if rank == 0:
+    if with_cpu:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    del path, W, x_full, x_host, y_full
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return line
+
+
+SUB_KEYS = ("value", "unit", "ms_per_step", "steps", "warmup", "config", "layer", "stack", "naive_pad", "route_cost",
+            "step0_truncated_after_detection", "prefix_kv_cache", "kernels", "roofline", "gpu_launches", "e2e",
+            "clocks", "cpu_baseline")
+
+
+def sub_record(line: dict) -> dict:
+    return {k: line[k] for k in SUB_KEYS if k in line}
+
+
+# ----------------------------------------------------------------- our arm
+def main():
+    args = parse()
+    suite = args.workload == "suite"
+    head = synth.workload(SUITE[0] if suite else int(args.workload))
+    if args.impl == "reference":
+        run_reference(args, head, int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), suite)
+        return
+    from paper_2607_14557_gb300 import seer as S_
+
+    S_.seer_set_launch_overlap(args.launch_overlap == "on")
+    env = Env()
+    with_cpu = env.world == 1 and env.rank == 0 and not args.no_cpu_baseline
+    run = run_stack if head.index == 3 else run_layer
+    line = run(args, head, env, with_cpu)
+    if suite:
+        line["config"]["suite"] = suite_note()
+        subs = {}
+        for idx in SUITE[1:]:
+            wl = synth.workload(idx)
+            rec = (run_stack if idx == 3 else run_layer)(args, wl, env, with_cpu)
+            subs[f"workload_{idx}"] = sub_record(rec)
+        line["sub_records"] = subs
+        line["gpu_launches_all_records"] = line["gpu_launches"] + sum(s["gpu_launches"] for s in subs.values())
+    if env.rank == 0:
         print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+    env.close()
 
 
 if __name__ == "__main__":

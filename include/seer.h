@@ -27,7 +27,10 @@
  *    three more mantissa bits) with fp32 accumulation.  A layer that stored
  *    its intermediates in bf16 misses |err| <= 1e-2 + 1e-2|ref| against the
  *    exact result on a few percent of outputs at d = 4096, F = 12288; with
- *    f16 intermediates it meets it.  Values must stay within the f16 range.
+ *    f16 intermediates it meets it.  Values must stay within the f16 range
+ *    (|v| <= 65504): every 16-bit store of the GEMM, attention and RMSNorm
+ *    kernels passes a range guard, and a value that overflowed to infinity
+ *    (or is NaN) records device error code 6, which seer_check_device reports.
  *  - There is no CPU fallback: without a usable GPU every call fails with
  *    SEER_ERR_CUDA.
  */
@@ -260,18 +263,23 @@ seer_status seer_swiglu(const void* a, const void* w_gate, const void* w_up, see
  * Same arguments and results as seer_attention, minus the workspace: the
  * schedule lives in a fixed 1 MiB __device__ array compiled into libseer,
  * held by every GPU that loads the library until the process exits.
- * n_heads * (ceil(T_capacity/128) + B) must stay <= 65504, else the call
- * returns SEER_ERR_WORKSPACE.  The first call on a device looks up the
- * array's device address (cudaGetSymbolAddress) with that device current,
- * so make it before any stream capture.  Allocates nothing.  Every call
- * reuses the same array: calls whose kernels overlap on the GPU race and must
- * not be issued (nothing in the array needs to start at zero). */
+ * For 16-bit attention n_heads * (ceil(T_capacity/128) + B) must stay
+ * <= 65520 (the work units whose schedule fits the array), else the call
+ * returns SEER_ERR_WORKSPACE; fp32 attention uses no schedule and has no such
+ * limit.  The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current, so make it before any
+ * stream capture; the address is kept for the process, so resetting the
+ * device (cudaDeviceReset) while libseer is loaded is not supported.
+ * Allocates nothing.  Every call reuses the same array: calls whose kernels
+ * overlap on the GPU race and must not be issued (nothing in the array needs
+ * to start at zero). */
 seer_status seer_attention_noalloc(const void* qkv, void* o, seer_dtype dt, const int32_t* cu_seqlens,
                                    const int32_t* kv_len, int B, int T_capacity, int n_heads, int head_dim,
                                    void* stream);
 
 /* dst[i] = src[i] converted (round to nearest even) for i < n; n % 8 == 0.
- * bf16 -> f16 is exact for |v| >= 2^-14 and below 65504 (f16's normal range).
+ * bf16 -> f16 is exact for |v| >= 2^-14 and below 65504 (f16's normal range);
+ * a 16-bit result that is infinite or NaN records device error code 6.
  * Used once per model to make the f16 weight copies of bf16 layers. */
 seer_status seer_convert(const void* src, seer_dtype src_dt, void* dst, seer_dtype dst_dt, size_t n, void* stream);
 
@@ -336,7 +344,9 @@ const char* seer_last_error(void);
 /* Synchronises the current device, then reports (and clears) the first
  * device-side error recorded by any kernel: SEER_OK or SEER_ERR_DEVICE with
  * code_out set (1 bad row count, 2 bad sequence layout, 3 pipeline wait timed
- * out, 4 boundary out of range, 5 capacity exceeded). */
+ * out, 4 boundary out of range, 5 capacity exceeded, 6 a stored 16-bit value
+ * is infinite or NaN: an f16 intermediate overflowed +-65504, or the input
+ * held a non-finite value). */
 seer_status seer_check_device(int* code_out);
 
 /* Failure-detection self-test: enqueues a kernel whose pipeline wait can

@@ -29,16 +29,25 @@ __device__ __forceinline__ void load8(const void* base, size_t i8, float (&v)[8]
     }
   }
 }
+// Stores 8 values; for 16-bit storage returns the range-guard terms of the
+// stored words (nonfinite_term), 0 for fp32.
 template <int T>
-__device__ __forceinline__ void store8(void* base, size_t i8, const float (&v)[8]) {
+__device__ __forceinline__ uint32_t store8(void* base, size_t i8, const float (&v)[8]) {
   if (T == kF32) {
     float4* p = reinterpret_cast<float4*>(base) + 2 * i8;
     p[0] = make_float4(v[0], v[1], v[2], v[3]);
     p[1] = make_float4(v[4], v[5], v[6], v[7]);
+    return 0u;
   } else {
-    reinterpret_cast<uint4*>(base)[i8] =
-        make_uint4(pack2(v[0], v[1], T == kF16), pack2(v[2], v[3], T == kF16), pack2(v[4], v[5], T == kF16),
-                   pack2(v[6], v[7], T == kF16));
+    uint32_t o[4];
+    uint32_t nf = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      o[k] = pack2(v[2 * k], v[2 * k + 1], T == kF16);
+      nf |= nonfinite_term(o[k], T == kF16);
+    }
+    reinterpret_cast<uint4*>(base)[i8] = make_uint4(o[0], o[1], o[2], o[3]);
+    return nf;
   }
 }
 
@@ -62,6 +71,7 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ x
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nwarps = gridDim.x * 8;
   const int d8 = d / 8;
+  uint32_t nonfinite = 0;
   for (int row = blockIdx.x * 8 + warp; row < M; row += nwarps) {
     const size_t base8 = static_cast<size_t>(row) * d8;
     float ss = 0.f;
@@ -80,9 +90,10 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ x
       load8<OUT>(g, v, gg);
 #pragma unroll
       for (int i = 0; i < 8; ++i) e[i] = e[i] * inv * gg[i];
-      store8<OUT>(y, base8 + v, e);
+      nonfinite |= store8<OUT>(y, base8 + v, e);
     }
   }
+  if (OUT != kF32) report_range(nonfinite, err);
 }
 
 // 16-bit rows of up to 256 * VPL elements: the row is read once into
@@ -112,6 +123,7 @@ __global__ void __launch_bounds__(256, 2) rmsnorm_rows_kernel(const void* __rest
   const uint4* xv = reinterpret_cast<const uint4*>(x);
   const uint4* gv = reinterpret_cast<const uint4*>(g);
   uint4* yv = reinterpret_cast<uint4*>(y);
+  uint32_t nonfinite = 0;
   for (int row = blockIdx.x * 8 + warp; row < M; row += nwarps) {
     const size_t base8 = static_cast<size_t>(row) * d8;
     uint4 raw[VPL];
@@ -143,25 +155,32 @@ __global__ void __launch_bounds__(256, 2) rmsnorm_rows_kernel(const void* __rest
         const uint32_t gw[4] = {gq.x, gq.y, gq.z, gq.w};
         uint32_t o[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
+        for (int k = 0; k < 4; ++k) {
           o[k] = pack2(lo16(w[k], IN == kF16) * inv * lo16(gw[k], OUT == kF16),
                        hi16(w[k], IN == kF16) * inv * hi16(gw[k], OUT == kF16), OUT == kF16);
+          nonfinite |= nonfinite_term(o[k], OUT == kF16);
+        }
         yv[base8 + v] = make_uint4(o[0], o[1], o[2], o[3]);
       }
     }
   }
+  report_range(nonfinite, err);
 }
 
-// Element-wise storage conversion (used once per model for f16 weight copies).
+// Element-wise storage conversion (used once per model for f16 weight copies);
+// a 16-bit result that is infinite or NaN (a bf16 weight beyond the f16
+// range) records kErrRange.
 template <int IN, int OUT>
-__global__ void convert_kernel(const void* __restrict__ src, void* __restrict__ dst, size_t n8) {
+__global__ void convert_kernel(const void* __restrict__ src, void* __restrict__ dst, size_t n8, int* err) {
   pdl_enter();
+  uint32_t nonfinite = 0;
   for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n8;
        i += static_cast<size_t>(gridDim.x) * blockDim.x) {
     float e[8];
     load8<IN>(src, i, e);
-    store8<OUT>(dst, i, e);
+    nonfinite |= store8<OUT>(dst, i, e);
   }
+  if (OUT != kF32) report_range(nonfinite, err);
 }
 
 // ------------------------------------------------------------------ rotary embedding
@@ -538,13 +557,13 @@ cudaError_t launch_rmsnorm(const void* x, int in_type, const void* g, void* y, i
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, cudaStream_t st) {
+cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, int* err, cudaStream_t st) {
   if (n == 0) return cudaSuccess;
   if (n % 8 != 0) return cudaErrorInvalidValue;
   const size_t n8 = n / 8;
   const int blocks = static_cast<int>(n8 / 256 + 1 < 4096 ? n8 / 256 + 1 : 4096);
 #define SEER_CONV(I, O) \
-  if (in_type == I && out_type == O) return launch_kernel(convert_kernel<I, O>, dim3(blocks), dim3(256), 0, st, src, dst, n8);
+  if (in_type == I && out_type == O) return launch_kernel(convert_kernel<I, O>, dim3(blocks), dim3(256), 0, st, src, dst, n8, err);
   SEER_CONV(kBF16, kF16)
   SEER_CONV(kF16, kBF16)
   SEER_CONV(kBF16, kF32)

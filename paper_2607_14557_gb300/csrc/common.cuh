@@ -22,10 +22,26 @@ enum DevErr : int {
   kErrTimeout = 3,     // a pipeline wait exceeded its time limit
   kErrBoundary = 4,    // L* outside [1, N]
   kErrCapacity = 5,    // packed rows exceed the output capacity
+  kErrRange = 6,       // a stored 16-bit value is infinite or NaN (an f16 intermediate beyond +-65504)
 };
 
 __device__ __forceinline__ void record_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
+}
+
+// Range guard of 16-bit stores.  For a word holding two f16 (or two bf16)
+// values, (v & exponent mask) + one unit of the exponent carries into a
+// half's top bit exactly when that half's exponent field is all ones, i.e.
+// the value is infinite or NaN (an f16 result of magnitude >= 65520 rounds to
+// infinity).  A thread ORs these terms over the words it stores -- three
+// integer operations per word -- and its warp reports once.
+__device__ __forceinline__ uint32_t nonfinite_term(uint32_t v, bool f16) {
+  return (v & (f16 ? 0x7C007C00u : 0x7F807F80u)) + (f16 ? 0x04000400u : 0x00800080u);
+}
+// Warp-collective: records kErrRange when any lane's accumulated terms flag a
+// non-finite store.
+__device__ __forceinline__ void report_range(uint32_t acc, int* err) {
+  if (__any_sync(0xffffffffu, (acc & 0x80008000u) != 0) && (threadIdx.x & 31) == 0) record_error(err, kErrRange);
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

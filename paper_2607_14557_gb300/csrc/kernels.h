@@ -75,6 +75,11 @@ int tc_attn_smem_bytes();
 // schedule from p.work_next until *p.work_count are done
 cudaError_t launch_tc_attn(const CUtensorMap& mQ, const CUtensorMap& mKV, const AttnParams& p, int grid, bool f16,
                            cudaStream_t st);
+// Bytes of schedule workspace the 16-bit attention kernels need for a launch
+// sized for T_cap rows, B segments and H heads: H * (ceil(T_cap/128) + B) work
+// units of 16 bytes, rounded up to 256 bytes, plus 256 bytes for the unit
+// count and the persistent kernel's unit counter.
+size_t attn_sched_bytes(int T_cap, int B, int H);
 // writes the units to work, their number to work_count[0] and zeroes
 // work_count[1] (the attention kernel's unit counter)
 cudaError_t launch_attn_schedule(const int* cu, const int* cu_kv, const int* kv_len, int B, int n_heads, int T_cap,
@@ -103,7 +108,7 @@ cudaError_t launch_resp_layout(const int* cu, const int* ctx, int B, int* cu_res
                                cudaStream_t st);
 // A bounded wait on a barrier that never completes (records kErrTimeout).
 cudaError_t launch_wait_selftest(uint64_t limit_ns, int* err, cudaStream_t st);
-cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, cudaStream_t st);
+cudaError_t launch_convert(const void* src, int in_type, void* dst, int out_type, size_t n, int* err, cudaStream_t st);
 cudaError_t launch_snr_scan(const int* counts, int B, int N, int F, double tau_jump, double gamma, int window,
                             int* L_star, int* i_star, cudaStream_t st);
 cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_full, const int* ctx_len,

@@ -182,10 +182,6 @@ struct LayerWs {
   size_t off_xn, off_qkv, off_h, off_act, off_sched, total;
 };
 
-size_t attn_sched_bytes(int T_cap, int B, int H) {
-  const size_t units = static_cast<size_t>(H) * (static_cast<size_t>((T_cap + 127) / 128) + static_cast<size_t>(B));
-  return align256(units * sizeof(int4)) + 256;
-}
 
 // Intermediates of one layer: fp32 for an fp32 layer, fp16 otherwise.
 LayerWs layer_ws(const seer_dims& d, seer_dtype dt, int T_cap, int B) {
@@ -428,9 +424,11 @@ seer_status do_attention(const void* qkv, void* o, seer_dtype dt, const int32_t*
     CUtensorMap m, mkv;
     SEER_TRY(make_map16(&m, qkv, dt, T_cap, 3 * H * dh, 3 * H * dh, 128));
     if (kvs.kv) SEER_TRY(make_map16(&mkv, kvs.kv, dt, kvs.T_kv_cap > 0 ? kvs.T_kv_cap : 1, kvs.ld, kvs.ld, 128));
-    Phase ph(PH_ATTN, st);
     SEER_CUDA(launch_attn_schedule(cu, p.cu_kv, kv_len, B, H, T_cap, work, count, max_units, di->err, st),
               "attn schedule");
+    // the attention phase brackets the attention kernel alone (the one-block
+    // schedule kernel before it takes a few microseconds)
+    Phase ph(PH_ATTN, st);
     // persistent: one CTA per SM (at most one per unit)
     SEER_CUDA(launch_tc_attn(m, kvs.kv ? mkv : m, p, std::min(max_units, di->num_sms), dt == SEER_F16, st),
               "tc_attn launch");
@@ -450,6 +448,11 @@ std::atomic<int> g_launch_overlap{1};
 }  // namespace
 
 namespace seer {
+size_t attn_sched_bytes(int T_cap, int B, int H) {
+  const size_t units = static_cast<size_t>(H) * (static_cast<size_t>((T_cap + 127) / 128) + static_cast<size_t>(B));
+  return ((units * sizeof(int4) + 255) & ~size_t(255)) + 256;
+}
+
 // Lets other translation units of the library report a message through
 // seer_last_error().
 void set_last_error(const char* msg) { g_msg = msg; }
@@ -544,7 +547,9 @@ seer_status seer_convert(const void* src, seer_dtype src_dt, void* dst, seer_dty
   if (!valid_dt(src_dt) || !valid_dt(dst_dt) || src_dt == dst_dt) return fail(SEER_ERR_INVALID_ARG, "convert: bad dtypes");
   if (n % 8 != 0) return fail(SEER_ERR_UNSUPPORTED, "convert: n must be a multiple of 8");
   if (!aligned16(src) || !aligned16(dst)) return fail(SEER_ERR_UNSUPPORTED, "convert: 16-byte aligned pointers required");
-  SEER_CUDA(launch_convert(src, src_dt, dst, dst_dt, n, static_cast<cudaStream_t>(stream)), "convert launch");
+  DeviceInfo* di;
+  SEER_TRY(device_info(&di));
+  SEER_CUDA(launch_convert(src, src_dt, dst, dst_dt, n, di->err, static_cast<cudaStream_t>(stream)), "convert launch");
   return SEER_OK;
 }
 

@@ -14,6 +14,8 @@
 // per device with cudaGetSymbolAddress on the first call made while that
 // device is current.  That first call therefore performs set-up and should
 // come before any CUDA stream capture.  No call allocates or frees memory.
+// The cached address belongs to the device's current context: resetting the
+// device (cudaDeviceReset) while libseer is loaded is not supported.
 //
 // All calls share the one array and leave their schedule in it.  Nothing in
 // it has to start at zero: the schedule kernel rewrites the entries and the
@@ -22,6 +24,7 @@
 #include <cuda_runtime.h>
 
 #include <cstddef>
+#include <cstdio>
 #include <mutex>
 
 #include "../../include/seer.h"
@@ -33,15 +36,15 @@ constexpr size_t kScratchBytes = size_t(1) << 20;
 
 static __device__ __align__(256) unsigned char g_attn_scratch[kScratchBytes];
 
+// Largest number of work units, n_heads * (ceil(T_capacity/128) + B), whose
+// schedule fits the array: units * 16 bytes rounded up to 256, plus 256 bytes
+// for the unit count and counter (65520 for 1 MiB).
+constexpr size_t kMaxUnits = (kScratchBytes - 256) / 16 / 16 * 16;
+static_assert(((kMaxUnits * 16 + 255) & ~size_t(255)) + 256 <= kScratchBytes, "limit must fit the array");
+static_assert((((kMaxUnits + 1) * 16 + 255) & ~size_t(255)) + 256 > kScratchBytes, "limit must be the largest");
+
 std::mutex g_mu;
 void* g_scratch_addr[64] = {};
-
-// Bytes of schedule the attention kernels use: H * (ceil(T/128) + B) int4
-// entries rounded up to 256 bytes, plus 256 bytes for the entry count.
-size_t schedule_bytes(int T_cap, int B, int H) {
-  const size_t units = static_cast<size_t>(H) * (static_cast<size_t>((T_cap + 127) / 128) + static_cast<size_t>(B));
-  return ((units * 16 + 255) & ~size_t(255)) + 256;
-}
 
 }  // namespace
 
@@ -52,11 +55,18 @@ extern "C" seer_status seer_attention_noalloc(const void* qkv, void* o, seer_dty
     seer::set_last_error("seer_attention_noalloc: bad sizes");
     return SEER_ERR_INVALID_ARG;
   }
-  const size_t need = schedule_bytes(T_capacity, B, n_heads);
+  // fp32 attention runs on CUDA cores without a schedule: nothing to hold
+  if (dt == SEER_F32)
+    return seer_attention(qkv, o, dt, cu_seqlens, kv_len, B, T_capacity, n_heads, head_dim, nullptr, 0, stream);
+  const size_t need = seer::attn_sched_bytes(T_capacity, B, n_heads);
   if (need > kScratchBytes) {
-    seer::set_last_error("seer_attention_noalloc: this batch needs a larger schedule than the built-in scratch "
-                         "of 1 MiB holds (n_heads * (ceil(T_capacity/128) + B) must stay <= 65504); use "
-                         "seer_attention with a caller-provided workspace");
+    char msg[256];
+    snprintf(msg, sizeof(msg),
+             "seer_attention_noalloc: this batch needs a larger schedule than the built-in scratch of 1 MiB holds "
+             "(n_heads * (ceil(T_capacity/128) + B) must stay <= %zu); use seer_attention with a caller-provided "
+             "workspace",
+             kMaxUnits);
+    seer::set_last_error(msg);
     return SEER_ERR_WORKSPACE;
   }
   int dev = 0;

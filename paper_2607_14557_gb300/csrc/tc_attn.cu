@@ -416,6 +416,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t tO = tmem + lane_off + TM_O + 128 * t;
     const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
     int cs = 0, co = 0, cv = 0;                   // S tiles seen, units done (this tile), V tiles before the unit
+    uint32_t nonfinite = 0;                       // range guard over this thread's output stores
     bool ok = true;
     for (int i = 0; ok; ++i) {
       const int u = __shfl_sync(0xffffffffu, read_unit(u_full, u_empty, unit_slot, i, abort_flag, p.err, lane == 0), 0);
@@ -531,10 +532,13 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint4* dst = reinterpret_cast<uint4*>(orow + 32 * cc);
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            dst[e] = make_uint4(pack2(__uint_as_float(rr[8 * e + 0]) * inv_l, __uint_as_float(rr[8 * e + 1]) * inv_l, F16),
-                                pack2(__uint_as_float(rr[8 * e + 2]) * inv_l, __uint_as_float(rr[8 * e + 3]) * inv_l, F16),
-                                pack2(__uint_as_float(rr[8 * e + 4]) * inv_l, __uint_as_float(rr[8 * e + 5]) * inv_l, F16),
-                                pack2(__uint_as_float(rr[8 * e + 6]) * inv_l, __uint_as_float(rr[8 * e + 7]) * inv_l, F16));
+            uint32_t q[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              q[k] = pack2(__uint_as_float(rr[8 * e + 2 * k]) * inv_l, __uint_as_float(rr[8 * e + 2 * k + 1]) * inv_l, F16);
+              nonfinite |= nonfinite_term(q[k], F16);
+            }
+            dst[e] = make_uint4(q[0], q[1], q[2], q[3]);
           }
         }
       }
@@ -544,6 +548,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       ++co;
       cv += d.nkv;
     }
+    report_range(nonfinite, p.err);               // an output value was infinite or NaN
   }
 
   tc_fence_before();
@@ -583,18 +588,16 @@ __global__ void attn_schedule_kernel(const int* cu, const int* cu_kv, const int*
     rank[i] = rk;
   }
   __syncthreads();
+  // offsets in rank order: a segment's units follow those of every segment
+  // ranked before it (the ranks are a permutation of 0..B-1)
+  for (int i = threadIdx.x; i < B; i += blockDim.x) {
+    int before = 0;
+    for (int k = 0; k < B; ++k) before += rank[k] < rank[i] ? ntile[k] : 0;
+    off[i] = H * before;
+  }
   if (threadIdx.x == 0) {
-    // walk segments in rank order accumulating offsets
     int acc = 0;
-    for (int rk = 0; rk < B; ++rk) {
-      for (int i = 0; i < B; ++i) {
-        if (rank[i] == rk) {
-          off[i] = acc;
-          acc += H * ntile[i];
-          break;
-        }
-      }
-    }
+    for (int i = 0; i < B; ++i) acc += H * ntile[i];
     if (acc > max_units) {
       record_error(err, kErrCapacity);
       acc = max_units;

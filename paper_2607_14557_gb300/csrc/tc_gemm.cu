@@ -26,6 +26,9 @@
 //   Count     detector: A rows gathered per sequence window, counts only
 //   Rope      Store, then the q|k columns rotated per 128-wide head by the
 //             rotary embedding at each row's position in its sequence
+// Every stored 16-bit value passes a range guard: an infinite or NaN result
+// (an f16 intermediate that overflowed +-65504) records kErrRange in the
+// device error word, which seer_check_device reports.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -237,6 +240,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     int acc = 0;
     uint32_t acc_ph = 0;
+    uint32_t nonfinite = 0;                      // range guard over this thread's stores
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
       int m, n;
       tile_coords(t, num_m, num_n, group_m, m, n);
@@ -278,14 +282,15 @@ __global__ void __launch_bounds__(THREADS, 1)
               }
 #pragma unroll
               for (int i = 0; i < 2; ++i) {
-                const float* w0 = v0 + 16 * i;
-                const float* w1 = v1 + 16 * i;
-                st_global_v8(crow + c0 + 16 * i, pack2(w0[0], w0[1], of16), pack2(w0[2], w0[3], of16),
-                             pack2(w0[4], w0[5], of16), pack2(w0[6], w0[7], of16), pack2(w0[8], w0[9], of16),
-                             pack2(w0[10], w0[11], of16), pack2(w0[12], w0[13], of16), pack2(w0[14], w0[15], of16));
-                st_global_v8(crow + c1 + 16 * i, pack2(w1[0], w1[1], of16), pack2(w1[2], w1[3], of16),
-                             pack2(w1[4], w1[5], of16), pack2(w1[6], w1[7], of16), pack2(w1[8], w1[9], of16),
-                             pack2(w1[10], w1[11], of16), pack2(w1[12], w1[13], of16), pack2(w1[14], w1[15], of16));
+                uint32_t q0[8], q1[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                  q0[e] = pack2(v0[16 * i + 2 * e], v0[16 * i + 2 * e + 1], of16);
+                  q1[e] = pack2(v1[16 * i + 2 * e], v1[16 * i + 2 * e + 1], of16);
+                  nonfinite |= nonfinite_term(q0[e], of16) | nonfinite_term(q1[e], of16);
+                }
+                st_global_v8(crow + c0 + 16 * i, q0[0], q0[1], q0[2], q0[3], q0[4], q0[5], q0[6], q0[7]);
+                st_global_v8(crow + c1 + 16 * i, q1[0], q1[1], q1[2], q1[3], q1[4], q1[5], q1[6], q1[7]);
               }
             }
           }
@@ -321,7 +326,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             uint32_t w[16];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) w[i] = pack2(v[2 * i], v[2 * i + 1], of16);
+            for (int i = 0; i < 16; ++i) {
+              w[i] = pack2(v[2 * i], v[2 * i + 1], of16);
+              nonfinite |= nonfinite_term(w[i], of16);
+            }
             if (slab_full) {
               store_chunk(w, n * BN + c * 32, m * BM + q * 32);
             } else {
@@ -376,7 +384,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (slab_full || store) {
               uint32_t w[16];
 #pragma unroll
-              for (int i = 0; i < 16; ++i) w[i] = pack2(a[2 * i], a[2 * i + 1], of16);
+              for (int i = 0; i < 16; ++i) {
+                w[i] = pack2(a[2 * i], a[2 * i + 1], of16);
+                nonfinite |= nonfinite_term(w[i], of16);
+              }
               if (slab_full) {
                 store_chunk(w, n * 128 + c * 32, m * BM + q * 32);
               } else {
@@ -393,6 +404,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (lane == 0) mbar_arrive(&acc_empty[acc]);
       if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
     }
+    report_range(nonfinite, p.err);              // a stored value overflowed the 16-bit type (or was NaN)
     if (lane == 0) bulk_wait_all();              // outputs written before the CTA exits
     __syncwarp();
   }

@@ -236,6 +236,24 @@ class SeerPath:
         kv = torch.as_tensor((ctx + L).astype(np.int32)).to(dev)
         return x, cu, kv, T
 
+    def varlen_only_inputs(self, x_full, cu_full, ctx_len, stream=None):
+        """The last step's batch packed with the static path switched off
+        (``tau_pad < 0``): every segment keeps exactly ``ctx_b + L*_b`` rows, so
+        no bucket padding is computed.  Compared with the routed layout it
+        prices the rows the static-graph groups pad (Sec. 3.4, Eq. 4).
+        Returns ``(x, cu, kv_len, T_capacity)``."""
+        B, dev = self.B, self.device
+        i32 = dict(dtype=torch.int32, device=dev)
+        x = torch.zeros_like(self.x_packed)
+        cu = torch.empty(B + 1, **i32)
+        kv = torch.empty(B, **i32)
+        meta = torch.empty(S.CTRL_WORDS, **i32)
+        p = self.params
+        no_static = S.make_params(p.act_eps, p.tau_jump, p.gamma, p.window, -1.0, p.eager_max_bucket, p.bucket_min)
+        S.seer_pack_ragged(x_full, self.dtype, cu_full, ctx_len, self.L_star, B, self.dims.d_model, self.N,
+                           self.T_full, no_static, x, cu, kv, meta, None, 0, stream=stream)
+        return x, cu, kv, self.T_full
+
     def padded_forward(self, x_full, cu_full, w: LayerWeights, y_full, stream=None):
         """The same layer over the untruncated windows (every key kept)."""
         S.seer_layer_forward(w.struct(), self.dims, self.dtype, x_full, y_full, cu_full, None, self.B, self.T_full,

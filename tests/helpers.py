@@ -8,6 +8,7 @@ BF16_ATOL = 1e-2
 BF16_RTOL = 1e-2
 F32_ATOL = 1e-4
 F32_RTOL = 1e-4
+COUNT_TOL_FRAC = 0.005    # near-zero counts within 0.5% of the intermediate width F
 
 
 def cuda():
@@ -50,6 +51,21 @@ def check_close(got, ref, dtype, what=""):
                              f"max err {np.nanmax(err):.4g}; first bad {idx.tolist()}; "
                              f"finite={np.isfinite(got).all()}")
     return float(err.max()) if err.size else 0.0
+
+
+def check_counts(got, ref, F, what=""):
+    """|got - ref| <= 0.5% of F for every token's near-zero count (the parity
+    bar of the sparsity counts); returns the largest difference."""
+    got = np.asarray(got, dtype=np.int64)
+    ref = np.asarray(ref, dtype=np.int64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    diff = np.abs(got - ref)
+    worst = int(diff.max()) if diff.size else 0
+    if worst > COUNT_TOL_FRAC * F:
+        idx = np.argwhere(diff > COUNT_TOL_FRAC * F)[:8]
+        raise AssertionError(f"{what}: max |count - oracle| = {worst} > {COUNT_TOL_FRAC * F:g} (0.5% of F={F}) at "
+                             f"{int((diff > COUNT_TOL_FRAC * F).sum())}/{diff.size} tokens; first {idx.tolist()}")
+    return worst
 
 
 def layer_weight_tensors(wl, w):

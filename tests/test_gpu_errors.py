@@ -114,3 +114,65 @@ def test_attention_segment_past_capacity_is_recorded_and_skipped():
     got = host(o)[:120].astype(np.float64)
     assert (np.abs(got - ref) <= 1e-2 + 1e-2 * np.abs(ref)).all()     # the valid segment still runs
     assert (host(o)[120:] == SENTINEL).all()                            # the bad one is skipped
+
+
+# ---------------------------------------------------------------- f16 range guard
+ERR_RANGE = 6
+
+
+def test_swiglu_intermediate_beyond_f16_range_is_recorded():
+    # a = SiLU(x Wg^T) * (x Wu^T) with x = 4 and weights 0.5 over K = 256: g = u = 512
+    # and a ~ 2.6e5, beyond f16's largest finite value 65504; the stored f16 `a` is
+    # infinite and the epilogue's range guard records the code.  The same call with
+    # x = 0.25 (a ~ 1024) stays finite and records nothing.
+    M, F, K = 256, 256, 256
+    wg = torch.full((F, K), 0.5, dtype=torch.float16, device=cuda())
+    wu = torch.full((F, K), 0.5, dtype=torch.float16, device=cuda())
+    act = torch.empty((M, F), dtype=torch.float16, device=cuda())
+    small = torch.full((M, K), 0.25, dtype=torch.float16, device=cuda())
+    S.seer_swiglu(small, wg, wu, "f16", act, "f16", M, None, F, K)
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == 0
+    assert torch.isfinite(act.float()).all()
+    big = torch.full((M, K), 4.0, dtype=torch.float16, device=cuda())
+    S.seer_swiglu(big, wg, wu, "f16", act, "f16", M, None, F, K)
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == ERR_RANGE
+    assert torch.isinf(act.float()).all()
+
+
+def test_layer_residual_beyond_f16_range_is_recorded():
+    # a bf16 layer whose input rows hold 1e5 (finite in bf16): the f16 residual
+    # stream h = x + o Wo^T overflows, and the O-projection epilogue records the
+    # code; the same layer on N(0, 1) rows records nothing
+    from tests.helpers import layer_weight_tensors, to_dev, weights_struct
+    import synth
+    wl = synth.tiny_workload(dtype="bf16", seed=410, d=256, n_heads=2, head_dim=128, d_ff=768, batch=2, window=64)
+    w = synth.layer_weights(wl, 0)
+    _, WL = layer_weight_tensors(wl, w)
+    dims = S.make_dims(wl.d, wl.n_heads, wl.head_dim, wl.d_ff)
+    T = 300
+    cu = i32([0, 140, T])
+    ws_bytes = S.seer_layer_workspace_size(dims, "bf16", T, 2)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=cuda())
+    y = torch.empty((T, wl.d), dtype=torch.bfloat16, device=cuda())
+    x = to_dev(np.random.default_rng(0).standard_normal((T, wl.d)), "bf16")
+    S.seer_layer_forward(weights_struct(WL), dims, "bf16", x, y, cu, None, 2, T, None, 0, 0.0, None, ws, ws_bytes)
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == 0
+    x_big = torch.full((T, wl.d), 1e5, dtype=torch.bfloat16, device=cuda())
+    S.seer_layer_forward(weights_struct(WL), dims, "bf16", x_big, y, cu, None, 2, T, None, 0, 0.0, None, ws, ws_bytes)
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == ERR_RANGE
+
+
+def test_convert_beyond_f16_range_is_recorded():
+    # bf16 -> f16 of 1e5 (finite in bf16, beyond f16) gives infinity and the code
+    src = torch.full((64,), 1e5, dtype=torch.bfloat16, device=cuda())
+    dst = torch.empty((64,), dtype=torch.float16, device=cuda())
+    S.seer_convert(src, "bf16", dst, "f16", 64)
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == ERR_RANGE
+    S.seer_convert(src / 4, "bf16", dst, "f16", 64)      # 25000: finite in f16
+    torch.cuda.synchronize()
+    assert S.seer_check_device() == 0

@@ -3,7 +3,9 @@
 
 The oracle cannot redo every row at these sizes, so it checks what it can
 compute one by one: every boundary (bit exact, planted), every packed row (bit
-exact), near-zero counts around every boundary, and the layer output of sampled
+exact), the near-zero counts of every token of whole windows (two or three
+sequences, every 128-row tile of the window) and around every other boundary,
+and the layer output of sampled
 query rows of the shortest and longest (and for workload 2 a middle) segment,
 with keys/values from all of that segment's kept rows.  Rows past the packed
 total must stay untouched.
@@ -14,7 +16,7 @@ import torch
 
 import oracle
 import synth
-from tests.helpers import check_close
+from tests.helpers import check_close, check_counts
 from tests.test_gpu_layer import run_path
 
 pytestmark = pytest.mark.gpu
@@ -51,13 +53,20 @@ def test_workload_full_size_sampled(index):
     assert (r["y"][T:] == 9.0).all()                # zero work past the packed total
     x, resp, w = r["x"], r["resp"], r["w"]
     F = wl.d_ff
-    for b in range(wl.batch):                       # counts around each boundary
-        bb = int(lens.boundary[b])
-        rows = np.arange(max(0, bb - 4), min(wl.window, bb + 5))
-        ref = oracle.sparsity_counts(x[resp[b] + rows], w["wg"], w["wu"], wl.act_eps)
-        assert np.abs(r["counts"][b, rows] - ref).max() <= 0.005 * F
-    rng = np.random.default_rng(index)
     order = np.argsort(seg)
+    # counts: every token of the whole window (all of its 128-row tiles) of the
+    # sequences with the shortest and longest kept segment (plus a middle one for
+    # workload 2), and around every other sequence's boundary
+    whole = {int(order[0]), int(order[-1])} | ({int(order[len(order) // 2])} if index == 2 else set())
+    for b in range(wl.batch):
+        if b in whole:
+            rows = np.arange(wl.window)
+        else:
+            bb = int(lens.boundary[b])
+            rows = np.arange(max(0, bb - 4), min(wl.window, bb + 5))
+        ref = oracle.sparsity_counts(x[resp[b] + rows], w["wg"], w["wu"], wl.act_eps)
+        check_counts(r["counts"][b, rows], ref, F, f"workload {index} window {b}")
+    rng = np.random.default_rng(index)
     picks = [order[0], order[-1]] + ([order[len(order) // 2]] if index == 2 else [])
     for b in picks:
         L = int(seg[b])
