@@ -41,6 +41,14 @@
 // Tensor memory (512 columns): S_0 | S_1 | O_0 | O_1, P_t packed into the
 // first 64 columns of S_t; a unit's first PV waits until the softmax warps
 // have read the previous unit's O_t out.
+//
+// Measured alternative, not adopted: 64-key sub-tiles with two 64-column score
+// buffers per tile, so the next QK^T runs during the softmax, were 11-16%
+// slower on GB300.  A QK^T of N = 64 reads its Q operand from shared memory at
+// the cost of one of N = 128 (the tensor core's shared-memory operand path
+// moves ~128 B/clk: M128 N64 K16 runs at 60% of the MMA rate alone, a 64-key
+// sub-tile's QK^T + PV at 82%), and beside the softmax's tensor-memory
+// traffic those MMAs ran at about half their isolated rate.
 #include <math.h>
 
 #include "common.cuh"
@@ -105,27 +113,46 @@ __device__ __forceinline__ float add_f16_hi(uint32_t v, float acc) {
   return d;
 }
 
+
+// Two fp32 fused multiply-adds in one instruction (packed f32x2, sm_100+).
+__device__ __forceinline__ void ffma2(float a0, float a1, float b0, float b1, float c0, float c1, float& d0, float& d1) {
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\t"
+      "mov.b64 rb, {%4, %5};\n\t"
+      "mov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\t"
+      "mov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+
 // Packed probabilities of keys 32c .. 32c+31 of one row: p = 2^(s * scale - m),
-// accumulated into the row sum.  f16: the exponent x is rounded to f16 and
-// two probabilities come from one MUFU operation (ex2.approx.f16x2) -- the
-// MUFU unit, not the tensor pipe, otherwise bounds a row's softmax; P is
-// stored in f16 anyway.  bf16: one fp32 ex2 per probability.
+// accumulated into the row sum.  f16: the exponents x of a pair come from one
+// packed f32x2 FMA, are rounded to f16, and two probabilities come from one
+// MUFU operation (ex2.approx.f16x2); P is stored in f16 anyway.  bf16: one
+// fp32 ex2 per probability.  Either way the row sum adds the stored (rounded)
+// probabilities.  The softmax of a tile sits on its tile's critical chain, so
+// its instruction count matters: the packed FMA is 2.5% faster on GB300, while
+// moving a quarter of the exponentials to a polynomial on the FMA pipes was 9%
+// slower (more instructions, no MUFU relief).
 template <bool F16>
 __device__ __forceinline__ void row_probs(const float* s, float scale_log2, float neg, float (&rs)[4],
                                           uint32_t (&pk)[16]) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
-    const float x0 = fmaf(s[2 * i], scale_log2, neg);
-    const float x1 = fmaf(s[2 * i + 1], scale_log2, neg);
     if (F16) {
+      float x0, x1;
+      ffma2(s[2 * i], s[2 * i + 1], scale_log2, scale_log2, neg, neg, x0, x1);
       const uint32_t ph = ex2_h2(pack_f16x2(x0, x1));
       rs[(2 * i) & 3] = add_f16_lo(ph, rs[(2 * i) & 3]);
       rs[(2 * i + 1) & 3] = add_f16_hi(ph, rs[(2 * i + 1) & 3]);
       pk[i] = ph;
     } else {
-      const float p0 = ex2(x0), p1 = ex2(x1);
-      rs[i & 3] += p0 + p1;
-      pk[i] = pack_bf16x2(p0, p1);
+      const float x0 = fmaf(s[2 * i], scale_log2, neg), x1 = fmaf(s[2 * i + 1], scale_log2, neg);
+      // the row sum adds the rounded probabilities the PV product reads, so
+      // numerator and normaliser carry the same rounding
+      const uint32_t ph = pack_bf16x2(ex2(x0), ex2(x1));
+      rs[i & 3] += bf16_lo(ph) + bf16_hi(ph);
+      pk[i] = ph;
     }
   }
 }
@@ -373,9 +400,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         // the first PV overwrites O_t: the previous unit's O_t must be read out
         if (oc > 0 && !mbar_wait(&o_free[t], (oc - 1) & 1u, abort_flag, p.err)) break;
         for (int j = 1; j < nkv; ++j) {
+          // operands first (usually landed long before), then this tile's P,
+          // then the turn: after P arrives only the turn is left to check
           if (!mbar_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err) ||
-              !mbar_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
               !mbar_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err) ||
+              !mbar_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
               (pair && !mbar_wait(&turn[t], tc & 1u, abort_flag, p.err))) {
             ok = false;
             break;
@@ -463,6 +492,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           for (int e = 0; e < w; ++e) mx[e] = fmaxf(mx[e], mx[e + w]);
         const float m_new = fmaxf(m_ref, mx[0] * scale_log2);
         const bool need = (j == 0) || (m_new > m_ref + RESCALE_THRESHOLD);
+        const bool any_need = __any_sync(0xffffffffu, need);
         float alpha = 1.f;
         if (need) {
           alpha = (j == 0) ? 0.f : ex2(m_ref - m_new);
@@ -480,7 +510,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         l = l * alpha + ((rs[0] + rs[1]) + (rs[2] + rs[3]));
         // rescale O_t in tensor memory if the reference max moved
-        if (j > 0 && __any_sync(0xffffffffu, need)) {
+        if (j > 0 && any_need) {
 #pragma unroll 1
           for (int cc = 0; cc < DH / 32; ++cc) {
             uint32_t rr[32];
