@@ -108,9 +108,10 @@ def measured_traffic(workload: int, phase: str):
         return None
     with open(path) as f:
         doc = json.load(f)
-    if code_digest(doc["sources"]) != doc.get("sources_code_sha1") or phase not in doc["kernels"]:
+    k = doc["kernels"].get(phase)
+    if k is None or code_digest(k["sources"]) != k.get("sources_code_sha1"):
         return None
-    return doc["kernels"][phase]["traffic_bytes"]
+    return k["traffic_bytes"]
 
 
 def graph_capacity(total: int) -> int:
