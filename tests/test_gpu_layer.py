@@ -315,3 +315,35 @@ def test_tiny_f16_model_path():
     ref = oracle.layer_forward_packed(host(xp)[:T], cu_ref, w, wl.n_heads, kv_len=kv_ref)
     check_close(host(y)[:T], ref, "bf16", "f16 model layer")
     assert (host(y)[T:] == 9.0).all()
+
+
+def test_varlen_only_inputs_repack_without_static_padding():
+    # the bench prices the static path's padding against this layout: the same batch
+    # re-packed with tau_pad < 0, every segment exactly ctx + L* rows (Sec. 3.4-3.5)
+    from paper_2607_14557_gb300 import driver as D
+    wl = synth.tiny_workload(dtype="bf16", seed=345, d=256, n_heads=2, head_dim=128, d_ff=768, batch=4, window=200,
+                             boundary=("uniform", 120, 127))
+    lens = synth.lengths(wl)
+    x, cu_full, resp = synth.hidden_full(wl, lens)
+    w = synth.layer_weights(wl, 0)
+    dims = S.make_dims(wl.d, wl.n_heads, wl.head_dim, wl.d_ff)
+    W = D.LayerWeights.from_host(w, "bf16")
+    path = D.SeerPath(dims, "bf16", wl.batch, wl.window, x.shape[0], S.make_params(wl.act_eps))
+    xd, cuf, ctx = to_dev(x, "bf16"), i32(cu_full), i32(lens.ctx)
+    path.step(xd, cuf, i32(resp), ctx, W)
+    route = path.route()
+    L = path.L_star.cpu().numpy()
+    assert route["pad_rows"] > 0                    # the routed layout pads a static group
+    xv, cuv, kvv, T_cap = path.varlen_only_inputs(xd, cuf, ctx)
+    torch.cuda.synchronize()
+    seg, kv, cu = oracle.segment_layout(lens.ctx, L, wl.window, -1.0)
+    np.testing.assert_array_equal(seg, lens.ctx + L)
+    np.testing.assert_array_equal(cuv.cpu().numpy(), cu)
+    np.testing.assert_array_equal(kvv.cpu().numpy(), kv)
+    T = int(cu[-1])
+    np.testing.assert_array_equal(host(xv)[:T], oracle.pack_rows(x, cu_full, seg))
+    y = torch.full((T_cap, wl.d), 9.0, dtype=torch.bfloat16, device=cuda())
+    path.layer(W, x=xv, y=y, cu=cuv, kv=kvv, T_cap=T_cap)
+    torch.cuda.synchronize()
+    ref = oracle.layer_forward_packed(host(xv)[:T], cu, w, wl.n_heads, kv_len=kv)
+    check_close(host(y)[:T], ref, "bf16", "varlen-only layer")
