@@ -718,6 +718,15 @@ def run_layer(args, wl, env, with_cpu):
                 "flops_per_launch": flops_of[dominant],
                 "why_this_kernel": "the tensor-core kernel with the largest share of the step's time "
                                    "(per-phase CUDA events)"}
+    if wl.dtype == "f32":
+        # the fp32 layer runs on CUDA cores: its gate/up GEMM against the fp32 FMA rate,
+        # derived from the unit counts and the clock (152 SMs x 128 fp32 lanes x 2 FLOP x 2.07 GHz)
+        alu_peak = 152 * 128 * 2 * 2.07e9 / 1e12
+        roofline.update({"kernel": "simt_gemm_kernel (gate/up + SwiGLU, fp32 CUDA cores)", "bound": "alu",
+                         "peak": alu_peak, "frac": achieved / alu_peak if achieved else None,
+                         "frac_of_sustained": None, "traffic": None,
+                         "peak_source": "derived: 152 SMs x 128 fp32 FMA lanes x 2 FLOP x 2.07 GHz (80.5 TFLOP/s)",
+                         "why_this_kernel": "the gate/up GEMM of the fp32 layer (latency-bound at ~121 rows)"})
 
     clocks = clk.summary()
     line = {
