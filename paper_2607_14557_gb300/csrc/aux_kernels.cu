@@ -384,7 +384,7 @@ __device__ __forceinline__ int graph_capacity(int total) {
 // Every block recomputes the (tiny) routing decision in shared memory, block 0
 // publishes it, then all blocks copy rows.  Dynamic smem: seg/cu/bucket-index
 // arrays of B+1 ints each.
-__global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restrict__ x_full, int row_bytes,
+__global__ void __launch_bounds__(256, 4) pack_route_kernel(const uint8_t* __restrict__ x_full, int row_bytes,
                                                          const int* __restrict__ cu_full,
                                                          const int* __restrict__ ctx_len,
                                                          const int* __restrict__ L_star, int B, int N, int T_cap,
@@ -473,28 +473,28 @@ __global__ void __launch_bounds__(256) pack_route_kernel(const uint8_t* __restri
   if (blockIdx.x == 0) {
     for (int i = threadIdx.x; i <= B; i += blockDim.x) cu_out[i] = cus[i];
     if (threadIdx.x == 0) {
-      int w[kCtrlWords];
-      for (int i = 0; i < kCtrlWords; ++i) w[i] = 0;
-      w[1] = rs.total;
-      w[2] = rs.max_seg;
-      w[3] = graph_capacity(rs.total);
-      w[4] = rs.n_groups;
-      w[5] = rs.path_mask;
-      w[6] = rs.pad_rows;
+      // the control word is assembled in place in meta_out (a local array of
+      // kCtrlWords ints would live on the stack and cost registers in every block)
+      for (int i = 0; i < kCtrlWords; ++i) meta_out[i] = 0;
+      meta_out[1] = rs.total;
+      meta_out[2] = rs.max_seg;
+      meta_out[3] = graph_capacity(rs.total);
+      meta_out[4] = rs.n_groups;
+      meta_out[5] = rs.path_mask;
+      meta_out[6] = rs.pad_rows;
       int g = 0;
       for (int k = 0; k < rs.n_buckets && g < kCtrlMaxGroups; ++k) {
         if (rs.count[k] == 0) continue;
-        w[8 + 4 * g + 0] = rs.bucket[k];
-        w[8 + 4 * g + 1] = rs.count[k];
-        w[8 + 4 * g + 2] = rs.path[k];
-        w[8 + 4 * g + 3] = rs.rho_ppm[k];
+        meta_out[8 + 4 * g + 0] = rs.bucket[k];
+        meta_out[8 + 4 * g + 1] = rs.count[k];
+        meta_out[8 + 4 * g + 2] = rs.path[k];
+        meta_out[8 + 4 * g + 3] = rs.rho_ppm[k];
         ++g;
       }
-      w[0] = epoch;
-      for (int i = 0; i < kCtrlWords; ++i) meta_out[i] = w[i];
+      meta_out[0] = epoch;
       if (host_ctrl != nullptr) {
         volatile int* hc = host_ctrl;
-        for (int i = 1; i < kCtrlWords; ++i) hc[i] = w[i];
+        for (int i = 1; i < kCtrlWords; ++i) hc[i] = meta_out[i];
         __threadfence_system();
         hc[0] = epoch;
         __threadfence_system();
@@ -628,8 +628,10 @@ cudaError_t launch_pack_route(const void* x_full, int elem_bytes, const int* cu_
                                          static_cast<int>(sm));
     if (e != cudaSuccess) return e;
   }
+  // four 256-thread blocks per SM are resident (64 registers): one wave, the warps
+  // looping over the rows
   int blocks = (T_cap + 7) / 8;
-  const int cap = num_sms * 8;
+  const int cap = num_sms * 4;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   return launch_kernel(pack_route_kernel, dim3(blocks), dim3(256), sm, st, reinterpret_cast<const uint8_t*>(x_full),
