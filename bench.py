@@ -55,8 +55,8 @@ KERNEL_OF_PHASE = {
     "gate_up": "tc_gemm_kernel<Swiglu> (gate/up + SwiGLU)",
     "down": "tc_gemm_kernel<Residual> (down projection + residual)",
 }
-# kept rows above which the oracle's layer time is scaled from a sample of
-# query rows instead of measured on every row
+# kept rows above which the oracle's layer time is extrapolated from a key/value
+# pass and a sample of query rows instead of measured on every row
 ORACLE_FULL_ROWS = 4096
 
 
@@ -196,11 +196,13 @@ def oracle_sample(wl):
     over its kept rows.
 
     Where the kept rows exceed ORACLE_FULL_ROWS (the video workload: ~12k rows,
-    about a minute of fp64 work), the layer runs on a sample of query rows (keys
-    and values still from every kept row) and its time is scaled to the whole
-    layer by the algorithmic FLOP count: K/V projections 4*keep*d^2 always,
-    plus per query row 4*d^2 (Q, O) + 6*d*F (MLP) + 4*d*keep (attention).  The
-    oracle is BLAS-bound, so its time follows the FLOPs.
+    about a minute of fp64 work), the layer time is extrapolated from two
+    measurements: the key/value pass over every kept row alone (RMSNorm and the
+    K and V projections, ``oracle.kv_prefill``: work the layer does once) and the
+    layer on a sample of n query rows (the same key/value pass plus, per query
+    row, its projections, attention over every key including the softmax's
+    exponentials, and the MLP).  The per-row part is the difference of the two,
+    scaled to every kept row: t = t_kv + (t_rows(n) - t_kv) * keep / n.
 
     Returns ``(kept_rows, seconds, description)``, seconds being the detection
     time plus the (possibly extrapolated) layer time."""
@@ -227,13 +229,14 @@ def oracle_sample(wl):
         n = 512
         q_rows = np.sort(np.random.default_rng(0).choice(keep, size=n, replace=False))
         t1 = time.perf_counter()
+        oracle.kv_prefill(seg, w, wl.n_heads)
+        t_kv = time.perf_counter() - t1
+        t1 = time.perf_counter()
         oracle.layer_forward_rows(seg, w, wl.n_heads, q_rows)
         t_n = time.perf_counter() - t1
-        d, F = wl.d, wl.d_ff
-        per_row = 4.0 * d * d + 6.0 * d * F + 4.0 * d * keep
-        t_layer = t_n * (4.0 * keep * d * d + keep * per_row) / (4.0 * keep * d * d + n * per_row)
-        how = (f"one truncated layer, scaled by FLOPs from {n} sampled query rows (keys/values from all {keep} "
-               f"rows; {t_n:.2f} s measured)")
+        t_layer = t_kv + max(t_n - t_kv, 0.0) * keep / n
+        how = (f"one truncated layer, extrapolated from the key/value pass over all {keep} rows ({t_kv:.2f} s) and the "
+               f"layer on {n} sampled query rows ({t_n:.2f} s): t_kv + (t_rows - t_kv) * {keep} / {n}")
     dt = t_detect + t_layer
     return keep, dt, (f"sequence {b} ({keep} kept rows of {int(lens.full[b])}): detection over its {wl.window}-token "
                       f"window + {how}, fp64 numpy")

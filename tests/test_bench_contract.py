@@ -30,8 +30,9 @@ def test_reference_arm_prints_the_contract_line():
 
 def test_reference_arm_suite_line_describes_the_headline_workload():
     # the default bench run leads with the video-shaped layer (workload 4): the
-    # reference arm reports the same config, its oracle sample scaled from sampled
-    # query rows (the ~12k-row layer would take about a minute of fp64 work)
+    # reference arm reports the same config, its oracle sample extrapolated from a
+    # key/value pass and sampled query rows (the ~12k-row layer would take about a
+    # minute of fp64 work)
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
                         "--warmup", "0"], capture_output=True, text=True, timeout=600, cwd=ROOT)
     assert r.returncode == 0, r.stderr[-2000:]
@@ -43,4 +44,4 @@ def test_reference_arm_suite_line_describes_the_headline_workload():
     assert cfg["batch"] == 4 and cfg["window"] == 2048
     assert cfg["route"]["pad_rows"] >= 0 and cfg["tokens_valid"] <= cfg["tokens_executed"] <= cfg["tokens_full"]
     assert d["value"] > 0 and d["cpu_baseline"]["value"] == d["value"]
-    assert "scaled by FLOPs" in d["cpu_baseline"]["sample"]
+    assert "extrapolated" in d["cpu_baseline"]["sample"]
