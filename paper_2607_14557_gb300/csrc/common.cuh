@@ -121,6 +121,11 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   return mbar_wait_for(bar, parity, abort, err, kWaitLimitNs);
 }
 
+// Bounded wait by every lane of a warp, with a warp-uniform outcome.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, err));
+}
+
 // Bounded wait used only while draining after an abort.
 __device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   const uint64_t t0 = globaltimer_ns();
@@ -147,6 +152,20 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 }
 
 // ---------------------------------------------------------------- tcgen05
+// One lane of a converged warp, chosen by elect.sync.  An MMA issuer written
+// as a whole warp that runs the issue loop in lockstep, with the elected lane
+// issuing, keeps its issue rate beside FMA-heavy warps on the same SM
+// sub-partition (GB300: the attention round's MMA stream at 99-100% of the
+// tensor rate); a lone lane in a divergent branch fell to 54-76% there.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t leader;
+  asm volatile(
+      "{\n\t.reg .pred P;\n\t"
+      "elect.sync _|P, 0xffffffff;\n\t"
+      "selp.u32 %0, 1, 0, P;\n\t}"
+      : "=r"(leader));
+  return leader != 0;
+}
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
                : "memory");

@@ -11,11 +11,11 @@
 // runs on across units, so a unit's Q / K loads and first QK^T overlap the
 // previous unit's last PV and epilogue (a CTA per unit paid ~3.4 us of
 // setup and teardown per unit, the persistent loop ~0.3 us).
-//   warp 0     TMA producers: lane 0 takes the next unit (atomic counter) and
+//   warp 0     TMA producer: takes the next unit (atomic counter) and
 //              publishes its index in a 4-entry shared ring, loads the unit's
-//              Q tiles once both issuers are done with the previous ones, and
-//              its K_j (2-deep ring); lane 1 loads V_j (2-deep ring); 128 keys
-//              x 128 dims with 128-byte swizzle;
+//              Q tiles once both issuers are done with the previous ones,
+//              then K_j and V_j in turn (two 2-deep rings); 128 keys x 128
+//              dims with 128-byte swizzle;
 //   warps 1-2  TMEM allocator (warp 1) and one MMA issuer per query tile t:
 //              O_t += P_t,j-1 V_j-1 (P from tensor memory, V an MN-major
 //              shared operand), then S_t,j = Q_t K_j^T (both from shared
@@ -32,6 +32,11 @@
 //              ring positions are unsigned counters (stage = c % 2, phase =
 //              c / 2 % 2).  A tile idle in a unit (odd tile count) only
 //              releases the Q, K and V stages it would have used;
+//              producer and issuers are whole warps running their loops in
+//              lockstep, one elected lane issuing (a lone lane in a divergent
+//              branch lost issue slots to the FMA-heavy softmax warps of its
+//              SM sub-partition, and the tensor pipe then ran at its pace:
+//              7-9% slower overall);
 //   warps 4-7  softmax of query tile 0, warps 8-11 of tile 1: one thread per
 //              query row holds the row's 128 scores, so no exchange between
 //              threads is needed.  While one group exponentiates its tile,
@@ -78,7 +83,7 @@ constexpr uint32_t TM_S = 0;                // S_t at TM_S + 128 t
 constexpr uint32_t TM_O = 256;              // O_t at TM_O + 128 t
 constexpr float RESCALE_THRESHOLD = 8.0f;   // log2 units
 constexpr int U_SLOTS = 4;                  // unit indices published ahead
-constexpr int U_READERS = 1 + NT + 4 * NT;   // V lane, NT issuers, 4 softmax warps per tile
+constexpr int U_READERS = NT + 4 * NT;       // NT issuers, 4 softmax warps per tile
 // barriers (8 bytes each), the unit ring, the TMEM base and the abort flag
 static_assert(8 * (2 + 2 * K_STAGES + 2 * V_STAGES + 5 * NT + 2 * U_SLOTS) + 4 * U_SLOTS + 8 <= 256,
               "barrier block");
@@ -254,93 +259,108 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    // -------------------------------------------------- TMA producers
-    // lane 0 takes the units from the global counter and loads each unit's
-    // Q tiles (once the previous unit's QK^T are done with them) and its K
-    // tiles; lane 1 loads the V tiles.  Both rings run on across the units
-    // of this CTA.
-    if (lane == 0) {
+    // -------------------------------------------------- TMA producer
+    // The whole warp runs the loop in lockstep (every wait by all lanes, with
+    // a warp-uniform outcome) and the elected lane issues: it takes the units
+    // from the global counter and publishes them in the shared ring, loads
+    // each unit's Q tiles (once the previous unit's QK^T are done with them),
+    // then its K_j and V_j in turn.  K_j needs the stage QK^T of round j-2
+    // released and V_j the stage PV of round j-2 (issued in round j-1)
+    // released, so one stream for both rings waits for nothing extra.  Both
+    // rings run on across the units of this CTA.
+    const bool leader = elect_one();
+    const int leader_lane = __ffs(__ballot_sync(0xffffffffu, leader)) - 1;
+    if (leader) {
       tma_prefetch_desc(&mQ);
       tma_prefetch_desc(&mKV);
-      int q_issued = 0, issued = 0;
-      bool ok = true;
-      int u = blockIdx.x;
-      unit_slot[0] = u;
+      unit_slot[0] = blockIdx.x;
       mbar_arrive(&u_full[0]);
-      for (int i = 0; ok && u >= 0; ++i) {
-        const Unit d = decode_unit(p, u);
-        if (i > 0 && !mbar_wait(q_empty, (i - 1) & 1, abort_flag, p.err)) break;
+    }
+    __syncwarp();
+    int q_issued = 0, k_issued = 0, v_issued = 0;
+    bool ok = true;
+    int u = blockIdx.x;
+    for (int i = 0; ok && u >= 0; ++i) {
+      const Unit d = decode_unit(p, u);
+      if (i > 0 && !warp_wait(q_empty, (i - 1) & 1, abort_flag, p.err)) break;
+      if (leader) {
         mbar_arrive_expect_tx(q_full, d.nt * TILE_BYTES);
         for (int t = 0; t < d.nt; ++t) {
           tma_load_2d(smem + OFF_Q + t * TILE_BYTES, &mQ, q_full, d.xq, d.q0 + t * BQ);
           tma_load_2d(smem + OFF_Q + t * TILE_BYTES + PANEL, &mQ, q_full, d.xq + 64, d.q0 + t * BQ);
         }
-        ++q_issued;
-        // publish unit i+1 now, so the V lane can run on into it
-        const int n = i + 1, sl = n % U_SLOTS;
-        if (n >= U_SLOTS && !mbar_wait(&u_empty[sl], (n / U_SLOTS - 1) & 1, abort_flag, p.err)) break;
-        int un = G + atomicAdd(p.work_next, 1);
+      }
+      __syncwarp();
+      ++q_issued;
+      // publish unit i+1 now, so the other roles can look ahead
+      const int n = i + 1, sl = n % U_SLOTS;
+      if (n >= U_SLOTS && !warp_wait(&u_empty[sl], (n / U_SLOTS - 1) & 1, abort_flag, p.err)) break;
+      int un = 0;
+      if (leader) {
+        un = G + atomicAdd(p.work_next, 1);
         if (un >= count) un = -1;
         unit_slot[sl] = un;
         mbar_arrive(&u_full[sl]);
-        for (int j = 0; j < d.nkv; ++j) {
-          const int st = issued % K_STAGES, use = issued / K_STAGES;
-          if (use > 0 && !mbar_wait(&k_empty[st], (use - 1) & 1, abort_flag, p.err)) { ok = false; break; }
-          uint8_t* dst = smem + OFF_K + st * TILE_BYTES;
-          mbar_arrive_expect_tx(&k_full[st], TILE_BYTES);
-          tma_load_2d(dst, &mKV, &k_full[st], d.xk, d.kv0 + j * BKV);
-          tma_load_2d(dst + PANEL, &mKV, &k_full[st], d.xk + 64, d.kv0 + j * BKV);
-          ++issued;
+      }
+      un = __shfl_sync(0xffffffffu, un, leader_lane);
+      for (int j = 0; j < d.nkv; ++j) {
+        const int ks = k_issued % K_STAGES, ku = k_issued / K_STAGES;
+        if (ku > 0 && !warp_wait(&k_empty[ks], (ku - 1) & 1, abort_flag, p.err)) { ok = false; break; }
+        if (leader) {
+          uint8_t* dst = smem + OFF_K + ks * TILE_BYTES;
+          mbar_arrive_expect_tx(&k_full[ks], TILE_BYTES);
+          tma_load_2d(dst, &mKV, &k_full[ks], d.xk, d.kv0 + j * BKV);
+          tma_load_2d(dst + PANEL, &mKV, &k_full[ks], d.xk + 64, d.kv0 + j * BKV);
         }
-        u = un;
-      }
-      if (*abort_flag) {
-        if (q_issued > 0) mbar_wait_drain(q_full, (q_issued - 1) & 1, 200000000ull);
-        for (int j = issued > K_STAGES ? issued - K_STAGES : 0; j < issued; ++j)
-          mbar_wait_drain(&k_full[j % K_STAGES], (j / K_STAGES) & 1, 200000000ull);
-      }
-    } else if (lane == 1) {
-      int issued = 0;
-      bool ok = true;
-      for (int i = 0; ok; ++i) {
-        const int u = read_unit(u_full, u_empty, unit_slot, i, abort_flag, p.err, true);
-        if (u < 0) break;
-        const Unit d = decode_unit(p, u);
-        for (int j = 0; j < d.nkv; ++j) {
-          const int st = issued % V_STAGES, use = issued / V_STAGES;
-          if (use > 0 && !mbar_wait(&v_empty[st], (use - 1) & 1, abort_flag, p.err)) { ok = false; break; }
-          uint8_t* dst = smem + OFF_V + st * TILE_BYTES;
-          mbar_arrive_expect_tx(&v_full[st], TILE_BYTES);
-          tma_load_2d(dst, &mKV, &v_full[st], d.xv, d.kv0 + j * BKV);
-          tma_load_2d(dst + PANEL, &mKV, &v_full[st], d.xv + 64, d.kv0 + j * BKV);
-          ++issued;
+        __syncwarp();
+        ++k_issued;
+        const int vs = v_issued % V_STAGES, vu = v_issued / V_STAGES;
+        if (vu > 0 && !warp_wait(&v_empty[vs], (vu - 1) & 1, abort_flag, p.err)) { ok = false; break; }
+        if (leader) {
+          uint8_t* dst = smem + OFF_V + vs * TILE_BYTES;
+          mbar_arrive_expect_tx(&v_full[vs], TILE_BYTES);
+          tma_load_2d(dst, &mKV, &v_full[vs], d.xv, d.kv0 + j * BKV);
+          tma_load_2d(dst + PANEL, &mKV, &v_full[vs], d.xv + 64, d.kv0 + j * BKV);
         }
+        __syncwarp();
+        ++v_issued;
       }
-      if (*abort_flag) {
-        for (int j = issued > V_STAGES ? issued - V_STAGES : 0; j < issued; ++j)
-          mbar_wait_drain(&v_full[j % V_STAGES], (j / V_STAGES) & 1, 200000000ull);
-      }
+      u = un;
+    }
+    if (*abort_flag && leader) {
+      // let copies still in flight land before the CTA's shared memory is released
+      if (q_issued > 0) mbar_wait_drain(q_full, (q_issued - 1) & 1, 200000000ull);
+      for (int j = k_issued > K_STAGES ? k_issued - K_STAGES : 0; j < k_issued; ++j)
+        mbar_wait_drain(&k_full[j % K_STAGES], (j / K_STAGES) & 1, 200000000ull);
+      for (int j = v_issued > V_STAGES ? v_issued - V_STAGES : 0; j < v_issued; ++j)
+        mbar_wait_drain(&v_full[j % V_STAGES], (j / V_STAGES) & 1, 200000000ull);
     }
   } else if (warp == 1 || warp == 2) {
+    // -------------------------------------------------- MMA issuer of tile t
+    // The whole warp runs the issue loop in lockstep (every wait by all lanes,
+    // with a warp-uniform outcome); the elected lane issues the MMAs, commits
+    // and arrivals.  A lone issuing lane in a divergent branch lost issue
+    // slots to the FMA-heavy softmax warps on its sub-partition, and the
+    // tensor pipe ran at its pace (84-94 cycles per 64-cycle MMA).
     const int t = warp - 1;
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer of tile t
-      constexpr uint32_t idesc_qk = make_idesc(BQ, BKV, 0, F16);
-      constexpr uint32_t idesc_pv = make_idesc(BQ, DH, 1, F16);
-      // descriptors built once; a K=16 step adds a constant to the
-      // start-address field (stage s of a ring: + s * TILE_BYTES / 16)
-      const uint64_t dq = make_sdesc_sw128(smem_u32(smem + OFF_Q + t * TILE_BYTES), 16, 1024);
-      const uint64_t dk0 = make_sdesc_sw128(smem_u32(smem + OFF_K), 16, 1024);
-      const uint64_t dv0 = make_sdesc_sw128(smem_u32(smem + OFF_V), PANEL, 1024);
-      const uint32_t dS = tmem + TM_S + 128 * t, dO = tmem + TM_O + 128 * t;
-      // ring positions run on across units: stage = count % 2, phase = count / 2 % 2
-      unsigned kc = 0, vc = 0;       // K / V tiles consumed
-      unsigned pc = 0, tc = 0;       // P tiles consumed, turn waits
-      unsigned oc = 0;               // units of this tile finished
-      bool paired_before = false;    // a unit with both tiles active was seen
-      bool ok = true;
-      // S_t = Q_t K^T for the K tile at ring position kc (both K-major, 128-byte swizzle)
-      auto qk = [&](unsigned c) {
+    const bool leader = elect_one();
+    constexpr uint32_t idesc_qk = make_idesc(BQ, BKV, 0, F16);
+    constexpr uint32_t idesc_pv = make_idesc(BQ, DH, 1, F16);
+    // descriptors built once; a K=16 step adds a constant to the
+    // start-address field (stage s of a ring: + s * TILE_BYTES / 16)
+    const uint64_t dq = make_sdesc_sw128(smem_u32(smem + OFF_Q + t * TILE_BYTES), 16, 1024);
+    const uint64_t dk0 = make_sdesc_sw128(smem_u32(smem + OFF_K), 16, 1024);
+    const uint64_t dv0 = make_sdesc_sw128(smem_u32(smem + OFF_V), PANEL, 1024);
+    const uint32_t dS = tmem + TM_S + 128 * t, dO = tmem + TM_O + 128 * t;
+    // ring positions run on across units: stage = count % 2, phase = count / 2 % 2
+    unsigned kc = 0, vc = 0;       // K / V tiles consumed
+    unsigned pc = 0, tc = 0;       // P tiles consumed, turn waits
+    unsigned oc = 0;               // units of this tile finished
+    bool paired_before = false;    // a unit with both tiles active was seen
+    bool ok = true;
+    // S_t = Q_t K^T for the K tile at ring position kc (both K-major, 128-byte swizzle)
+    auto qk = [&](unsigned c) {
+      if (leader) {
         const uint64_t dk = dk0 + static_cast<uint64_t>((c & 1u) * (TILE_BYTES >> 4));
 #pragma unroll
         for (int k = 0; k < DH / 16; ++k) {
@@ -349,91 +369,100 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         tc_commit(&s_full[t]);
         tc_commit(&k_empty[c & 1u]);
-      };
-      // O_t (+)= P_t V for the V tile at ring position c: A = P from tensor
-      // memory (8 columns per 16 keys), B = V [keys, dims] with dims
-      // contiguous, an MN-major operand whose 64-dim panels are PANEL bytes
-      // apart (LBO) and 8-key groups 1 KB apart (SBO)
-      // (vt: the V tile's index in the unit; tile 0 starts a fresh O_t)
-      auto pv = [&](unsigned c, int vt) {
+      }
+      __syncwarp();
+    };
+    // O_t (+)= P_t V for the V tile at ring position c: A = P from tensor
+    // memory (8 columns per 16 keys), B = V [keys, dims] with dims
+    // contiguous, an MN-major operand whose 64-dim panels are PANEL bytes
+    // apart (LBO) and 8-key groups 1 KB apart (SBO)
+    // (vt: the V tile's index in the unit; tile 0 starts a fresh O_t)
+    auto pv = [&](unsigned c, int vt) {
+      if (leader) {
         const uint64_t dv = dv0 + static_cast<uint64_t>((c & 1u) * (TILE_BYTES >> 4));
 #pragma unroll
         for (int k = 0; k < BKV / 16; ++k)
           tc_mma_f16_tmem_a(dO, dS + 8 * k, dv + static_cast<uint64_t>(k * 128), idesc_pv, (vt > 0 || k > 0) ? 1u : 0u);
         tc_commit(&v_empty[c & 1u]);
-      };
-      for (int i = 0; ok; ++i) {
-        const int u = read_unit(u_full, u_empty, unit_slot, i, abort_flag, p.err, true);
-        if (u < 0) break;
-        const Unit d = decode_unit(p, u);
-        if (!mbar_wait(q_full, i & 1, abort_flag, p.err)) break;
-        if (t >= d.nt) {
-          // idle this unit: release Q and every K / V stage as they pass
-          mbar_arrive(q_empty);
-          for (int j = 0; j < d.nkv; ++j, ++kc, ++vc) {
-            if (!mbar_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err) ||
-                !mbar_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err)) {
-              ok = false;
-              break;
-            }
-            mbar_arrive(&k_empty[kc & 1u]);
-            mbar_arrive(&v_empty[vc & 1u]);
-          }
-          continue;
-        }
-        const bool pair = d.nt > 1;
-        const int nkv = d.nkv;
-        // rounds: 0 = QK^T of K_0; j = 1 .. nkv-1: PV of V_j-1, then QK^T of
-        // K_j; nkv = PV of V_nkv-1.  Round j of tile 1 follows round j of tile
-        // 0, which follows round j-1 of tile 1 (the turn token); tile 0's
-        // round 0 follows tile 1's last round of the previous paired unit.
-        if (!mbar_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err)) break;
-        if (pair && (t == 1 || paired_before)) {
-          if (!mbar_wait(&turn[t], tc & 1u, abort_flag, p.err)) break;
-          ++tc;
-        }
-        tc_fence_after();
-        qk(kc);
-        ++kc;
-        if (nkv == 1) tc_commit(q_empty);
-        if (pair) mbar_arrive(&turn[t ^ 1]);
-        // the first PV overwrites O_t: the previous unit's O_t must be read out
-        if (oc > 0 && !mbar_wait(&o_free[t], (oc - 1) & 1u, abort_flag, p.err)) break;
-        for (int j = 1; j < nkv; ++j) {
-          // operands first (usually landed long before), then this tile's P,
-          // then the turn: after P arrives only the turn is left to check
-          if (!mbar_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err) ||
-              !mbar_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err) ||
-              !mbar_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
-              (pair && !mbar_wait(&turn[t], tc & 1u, abort_flag, p.err))) {
+      }
+      __syncwarp();
+    };
+    auto arrive = [&](uint64_t* bar) {
+      if (leader) mbar_arrive(bar);
+      __syncwarp();
+    };
+    for (int i = 0; ok; ++i) {
+      const int u = __shfl_sync(0xffffffffu, read_unit(u_full, u_empty, unit_slot, i, abort_flag, p.err, lane == 0), 0);
+      if (u < 0) break;
+      const Unit d = decode_unit(p, u);
+      if (!warp_wait(q_full, i & 1, abort_flag, p.err)) break;
+      if (t >= d.nt) {
+        // idle this unit: release Q and every K / V stage as they pass
+        arrive(q_empty);
+        for (int j = 0; j < d.nkv; ++j, ++kc, ++vc) {
+          if (!warp_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err) ||
+              !warp_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err)) {
             ok = false;
             break;
           }
-          tc += pair ? 1u : 0u;
-          tc_fence_after();
-          pv(vc, j - 1);
-          qk(kc);
-          ++vc;
-          ++pc;
-          ++kc;
-          if (pair) mbar_arrive(&turn[t ^ 1]);
+          arrive(&k_empty[kc & 1u]);
+          arrive(&v_empty[vc & 1u]);
         }
-        if (!ok) break;
-        if (nkv > 1) tc_commit(q_empty);
-        if (!mbar_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err) ||
-            !mbar_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
-            (pair && !mbar_wait(&turn[t], tc & 1u, abort_flag, p.err)))
+        continue;
+      }
+      const bool pair = d.nt > 1;
+      const int nkv = d.nkv;
+      // rounds: 0 = QK^T of K_0; j = 1 .. nkv-1: PV of V_j-1, then QK^T of
+      // K_j; nkv = PV of V_nkv-1.  Round j of tile 1 follows round j of tile
+      // 0, which follows round j-1 of tile 1 (the turn token); tile 0's
+      // round 0 follows tile 1's last round of the previous paired unit.
+      if (!warp_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err)) break;
+      if (pair && (t == 1 || paired_before)) {
+        if (!warp_wait(&turn[t], tc & 1u, abort_flag, p.err)) break;
+        ++tc;
+      }
+      tc_fence_after();
+      qk(kc);
+      ++kc;
+      if (nkv == 1 && leader) tc_commit(q_empty);
+      if (pair) arrive(&turn[t ^ 1]);
+      // the first PV overwrites O_t: the previous unit's O_t must be read out
+      if (oc > 0 && !warp_wait(&o_free[t], (oc - 1) & 1u, abort_flag, p.err)) break;
+      for (int j = 1; j < nkv; ++j) {
+        // operands first (usually landed long before), then this tile's P,
+        // then the turn: after P arrives only the turn is left to check
+        if (!warp_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err) ||
+            !warp_wait(&k_full[kc & 1u], (kc >> 1) & 1u, abort_flag, p.err) ||
+            !warp_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
+            (pair && !warp_wait(&turn[t], tc & 1u, abort_flag, p.err))) {
+          ok = false;
           break;
+        }
         tc += pair ? 1u : 0u;
         tc_fence_after();
-        pv(vc, nkv - 1);
-        tc_commit(&o_done[t]);
+        pv(vc, j - 1);
+        qk(kc);
         ++vc;
         ++pc;
-        if (pair) mbar_arrive(&turn[t ^ 1]);
-        if (pair) paired_before = true;
-        ++oc;
+        ++kc;
+        if (pair) arrive(&turn[t ^ 1]);
       }
+      if (!ok) break;
+      if (nkv > 1 && leader) tc_commit(q_empty);
+      if (!warp_wait(&v_full[vc & 1u], (vc >> 1) & 1u, abort_flag, p.err) ||
+          !warp_wait(&p_full[t], pc & 1u, abort_flag, p.err) ||
+          (pair && !warp_wait(&turn[t], tc & 1u, abort_flag, p.err)))
+        break;
+      tc += pair ? 1u : 0u;
+      tc_fence_after();
+      pv(vc, nkv - 1);
+      if (leader) tc_commit(&o_done[t]);
+      __syncwarp();
+      ++vc;
+      ++pc;
+      if (pair) arrive(&turn[t ^ 1]);
+      if (pair) paired_before = true;
+      ++oc;
     }
   } else if (warp >= 4) {
     // -------------------------------------------------- softmax warps 4..11

@@ -6,9 +6,11 @@
 // One CTA per SM, 192 threads, warp-specialised:
 //   warp 0      TMA producer: 128x64 A tile + two 128x64 B tiles per stage
 //               (128-byte swizzle), 4-stage ring of 48 KB stages;
-//   warp 1      TMEM allocator + single-thread MMA issuer: 4 x
-//               tcgen05.mma (M=128, N=256, K=16) per stage into one of two
-//               256-column fp32 accumulators (double buffered, 512 columns);
+//   warp 1      TMEM allocator + MMA issuer: 4 x tcgen05.mma (M=128, N=256,
+//               K=16) per stage into one of two 256-column fp32
+//               accumulators (double buffered, 512 columns);
+//               producer and issuer are whole warps in lockstep, one elected
+//               lane issuing;
 //   warps 2-5   epilogue: tcgen05.ld of the accumulator (each warp owns one
 //               32-lane quarter of TMEM = 32 output rows), fused epilogue,
 //               32 x 32 output chunks staged in shared memory and written by
@@ -130,65 +132,74 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
-    if (lane == 0) {
-      // ------------------------------------------------ TMA producer
+    // ------------------------------------------------ TMA producer
+    // Producer and issuer run as whole warps in lockstep (every wait by all
+    // lanes, with a warp-uniform outcome); the elected lane issues the copies
+    // and MMAs.  A lone lane in a divergent branch loses issue slots to the
+    // FMA-heavy epilogue warp on its SM sub-partition.
+    const bool leader = elect_one();
+    if (leader) {
       tma_prefetch_desc(&mA);
       tma_prefetch_desc(&mB0);
       tma_prefetch_desc(&mB1);
-      int s = 0;
-      uint32_t ph = 0;
-      long issued = 0;
-      for (int t = blockIdx.x; t < num_tiles && !*abort_flag; t += gridDim.x) {
-        int m, n;
-        tile_coords(t, num_m, num_n, group_m, m, n);
-        int a_row;
-        if (MODE == kGemmCount) {
-          const int b = m / tiles_per_seq;
-          const int j = m - b * tiles_per_seq;
-          const int rs = p.resp_start[b];
-          if (rs < 0 || rs + p.Nw > p.M_cap) record_error(p.err, kErrLayout);
-          a_row = rs + j * BM;
-        } else {
-          a_row = m * BM;
-        }
-        const int b_row0 = halfN ? n * 128 : n * BN;
-        const int b_row1 = halfN ? n * 128 : n * BN + 128;
-        bool ok = true;
-        for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.err)) { ok = false; break; }
+    }
+    int s = 0;
+    uint32_t ph = 0;
+    long issued = 0;
+    for (int t = blockIdx.x; t < num_tiles && !__any_sync(0xffffffffu, *abort_flag != 0); t += gridDim.x) {
+      int m, n;
+      tile_coords(t, num_m, num_n, group_m, m, n);
+      int a_row;
+      if (MODE == kGemmCount) {
+        const int b = m / tiles_per_seq;
+        const int j = m - b * tiles_per_seq;
+        const int rs = p.resp_start[b];
+        if (leader && (rs < 0 || rs + p.Nw > p.M_cap)) record_error(p.err, kErrLayout);
+        a_row = rs + j * BM;
+      } else {
+        a_row = m * BM;
+      }
+      const int b_row0 = halfN ? n * 128 : n * BN;
+      const int b_row1 = halfN ? n * 128 : n * BN + 128;
+      bool ok = true;
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!warp_wait(&empty[s], ph ^ 1u, abort_flag, p.err)) { ok = false; break; }
+        if (leader) {
           uint8_t* sa = smem + s * STAGE_BYTES;
           mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
           tma_load_2d(sa, &mA, &full[s], kb * BK, a_row);
           tma_load_2d(sa + A_TILE_BYTES, &mB0, &full[s], kb * BK, b_row0);
           tma_load_2d(sa + A_TILE_BYTES + B_HALF_BYTES, &mB1, &full[s], kb * BK, b_row1);
-          ++issued;
-          if (++s == STAGES) { s = 0; ph ^= 1u; }
         }
-        if (!ok) break;
+        __syncwarp();
+        ++issued;
+        if (++s == STAGES) { s = 0; ph ^= 1u; }
       }
-      if (*abort_flag) {
-        // let copies still in flight land before the CTA's shared memory is released
-        const long first = issued > STAGES ? issued - STAGES : 0;
-        for (long i = first; i < issued; ++i)
-          mbar_wait_drain(&full[i % STAGES], static_cast<uint32_t>((i / STAGES) & 1), 200000000ull);
-      }
+      if (!ok) break;
+    }
+    if (*abort_flag && leader) {
+      // let copies still in flight land before the CTA's shared memory is released
+      const long first = issued > STAGES ? issued - STAGES : 0;
+      for (long i = first; i < issued; ++i)
+        mbar_wait_drain(&full[i % STAGES], static_cast<uint32_t>((i / STAGES) & 1), 200000000ull);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
-      const uint32_t idesc = p.idesc;
-      int s = 0;
-      uint32_t ph = 0;
-      int acc = 0;
-      uint32_t acc_ph = 0;
-      for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        if (!mbar_wait(&acc_empty[acc], acc_ph ^ 1u, abort_flag, p.err)) break;
+    // ------------------------------------------------ MMA issuer
+    const bool leader = elect_one();
+    const uint32_t idesc = p.idesc;
+    int s = 0;
+    uint32_t ph = 0;
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+      if (!warp_wait(&acc_empty[acc], acc_ph ^ 1u, abort_flag, p.err)) break;
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * ACC_COLS);
+      bool ok = true;
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!warp_wait(&full[s], ph, abort_flag, p.err)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * ACC_COLS);
-        bool ok = true;
-        for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&full[s], ph, abort_flag, p.err)) { ok = false; break; }
-          tc_fence_after();
+        if (leader) {
           const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
           const uint64_t adesc = make_sdesc_sw128(sa, 16, 1024);
           const uint64_t bdesc = make_sdesc_sw128(sa + A_TILE_BYTES, 16, 1024);
@@ -198,14 +209,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc_mma_f16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
           }
           tc_commit(&empty[s]);
-          if (++s == STAGES) { s = 0; ph ^= 1u; }
         }
-        if (!ok) break;
-        tc_commit(&acc_full[acc]);
-        if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
+        __syncwarp();
+        if (++s == STAGES) { s = 0; ph ^= 1u; }
       }
-      pdl_trigger();                             // last MMAs issued: the next kernel may launch
+      if (!ok) break;
+      if (leader) tc_commit(&acc_full[acc]);
+      __syncwarp();
+      if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
     }
+    if (leader) pdl_trigger();                   // last MMAs issued: the next kernel may launch
   } else {
     // -------------------------------------------------- epilogue warps 2..5
     const int q = warp & 3;                    // TMEM lane quarter owned by this warp
