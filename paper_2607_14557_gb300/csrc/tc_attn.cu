@@ -36,7 +36,10 @@
 //              lockstep, one elected lane issuing (a lone lane in a divergent
 //              branch lost issue slots to the FMA-heavy softmax warps of its
 //              SM sub-partition, and the tensor pipe then ran at its pace:
-//              7-9% slower overall);
+//              7-9% slower overall).  A round's PV goes out in two halves of
+//              64 keys as the softmax warps release the halves of P_t, so the
+//              first half's MMAs overlap the second half's exponentials
+//              (5-8% faster);
 //   warps 4-7  softmax of query tile 0, warps 8-11 of tile 1: one thread per
 //              query row holds the row's 128 scores, so no exchange between
 //              threads is needed.  While one group exponentiates its tile,
@@ -76,7 +79,8 @@ constexpr int OFF_Q = 0;                                   // Q tiles 0, 1
 constexpr int OFF_K = NT * TILE_BYTES;
 constexpr int OFF_V = OFF_K + K_STAGES * TILE_BYTES;
 constexpr int OFF_BAR = OFF_V + V_STAGES * TILE_BYTES;
-constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+constexpr int BAR_BYTES = 512;
+constexpr int SMEM_BYTES = OFF_BAR + BAR_BYTES + 1024;
 static_assert(SMEM_BYTES <= 232448, "shared memory per CTA");
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t TM_S = 0;                // S_t at TM_S + 128 t
@@ -85,7 +89,7 @@ constexpr float RESCALE_THRESHOLD = 8.0f;   // log2 units
 constexpr int U_SLOTS = 4;                  // unit indices published ahead
 constexpr int U_READERS = NT + 4 * NT;       // NT issuers, 4 softmax warps per tile
 // barriers (8 bytes each), the unit ring, the TMEM base and the abort flag
-static_assert(8 * (2 + 2 * K_STAGES + 2 * V_STAGES + 5 * NT + 2 * U_SLOTS) + 4 * U_SLOTS + 8 <= 256,
+static_assert(8 * (2 + 2 * K_STAGES + 2 * V_STAGES + 6 * NT + 2 * U_SLOTS) + 4 * U_SLOTS + 8 <= BAR_BYTES,
               "barrier block");
 
 __device__ __forceinline__ float ex2(float x) {
@@ -214,8 +218,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint64_t* v_full = k_empty + K_STAGES;     // [V_STAGES]
   uint64_t* v_empty = v_full + V_STAGES;     // [V_STAGES]
   uint64_t* s_full = v_empty + V_STAGES;     // [NT] S_t,j written (and O_t += P_t,j-1 V done)
-  uint64_t* p_full = s_full + NT;            // [NT] P_t,j in tensor memory (O_t rescaled)
-  uint64_t* o_done = p_full + NT;            // [NT] last PV of tile t of a unit complete
+  uint64_t* p_full = s_full + NT;            // [NT] P_t,j of keys 0..63 in tensor memory (O_t rescaled)
+  uint64_t* p_full2 = p_full + NT;           // [NT] P_t,j of keys 64..127 in tensor memory
+  uint64_t* o_done = p_full2 + NT;           // [NT] last PV of tile t of a unit complete
   uint64_t* o_free = o_done + NT;            // [NT] O_t of a unit read out by the softmax warps
   uint64_t* turn = o_free + NT;              // [NT] issuer t may enqueue its next round
   uint64_t* u_full = turn + NT;              // [U_SLOTS] unit index published
@@ -241,6 +246,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     for (int t = 0; t < NT; ++t) {
       mbar_init(&s_full[t], 1);
       mbar_init(&p_full[t], 4);
+      mbar_init(&p_full2[t], 4);
       mbar_init(&o_done[t], 1);
       mbar_init(&o_free[t], 4);
       mbar_init(&turn[t], 1);
@@ -376,14 +382,18 @@ __global__ void __launch_bounds__(THREADS, 1)
     // memory (8 columns per 16 keys), B = V [keys, dims] with dims
     // contiguous, an MN-major operand whose 64-dim panels are PANEL bytes
     // apart (LBO) and 8-key groups 1 KB apart (SBO)
-    // (vt: the V tile's index in the unit; tile 0 starts a fresh O_t)
-    auto pv = [&](unsigned c, int vt) {
+    // (vt: the V tile's index in the unit; tile 0 starts a fresh O_t).
+    // Issued in two halves of 64 keys, each once the softmax warps have
+    // released that half of P_t.
+    auto pv = [&](unsigned c, int vt, int half) {
       if (leader) {
         const uint64_t dv = dv0 + static_cast<uint64_t>((c & 1u) * (TILE_BYTES >> 4));
 #pragma unroll
-        for (int k = 0; k < BKV / 16; ++k)
+        for (int kk = 0; kk < BKV / 32; ++kk) {
+          const int k = half * (BKV / 32) + kk;
           tc_mma_f16_tmem_a(dO, dS + 8 * k, dv + static_cast<uint64_t>(k * 128), idesc_pv, (vt > 0 || k > 0) ? 1u : 0u);
-        tc_commit(&v_empty[c & 1u]);
+        }
+        if (half == 1) tc_commit(&v_empty[c & 1u]);
       }
       __syncwarp();
     };
@@ -440,7 +450,13 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         tc += pair ? 1u : 0u;
         tc_fence_after();
-        pv(vc, j - 1);
+        pv(vc, j - 1, 0);
+        if (!warp_wait(&p_full2[t], pc & 1u, abort_flag, p.err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        pv(vc, j - 1, 1);
         qk(kc);
         ++vc;
         ++pc;
@@ -455,7 +471,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       tc += pair ? 1u : 0u;
       tc_fence_after();
-      pv(vc, nkv - 1);
+      pv(vc, nkv - 1, 0);
+      if (!warp_wait(&p_full2[t], pc & 1u, abort_flag, p.err)) break;
+      tc_fence_after();
+      pv(vc, nkv - 1, 1);
       if (leader) tc_commit(&o_done[t]);
       __syncwarp();
       ++vc;
@@ -528,51 +547,61 @@ __global__ void __launch_bounds__(THREADS, 1)
           m_ref = m_new;
         }
         // P_t,j: keys 32c .. 32c+31 -> 16 packed columns 16c .. 16c+15 of S_t
-        // (the scores were all read above; O_t += P_t,j-1 V_j-1 has completed)
+        // (the scores were all read above; O_t += P_t,j-1 V_j-1 has completed),
+        // released to the PV MMAs in two halves of 64 keys, so the first
+        // half's MMAs run while the second half is exponentiated
         const float neg = -m_ref;
         float rs[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int cc = 0; cc < BKV / 32; ++cc) {
-          uint32_t pk[16];
-          row_probs<F16>(s + 32 * cc, scale_log2, neg, rs, pk);
-          tmem_st16(tS + 16 * cc, pk);
-        }
-        l = l * alpha + ((rs[0] + rs[1]) + (rs[2] + rs[3]));
-        // rescale O_t in tensor memory if the reference max moved
-        if (j > 0 && any_need) {
+        for (int hf = 0; hf < 2; ++hf) {
+#pragma unroll
+          for (int cc = 2 * hf; cc < 2 * hf + 2; ++cc) {
+            uint32_t pk[16];
+            row_probs<F16>(s + 32 * cc, scale_log2, neg, rs, pk);
+            tmem_st16(tS + 16 * cc, pk);
+          }
+          if (hf == 0) {
+            // before the first half is released: rescale O_t in tensor memory
+            // if the reference max moved ...
+            if (j > 0 && any_need) {
 #pragma unroll 1
-          for (int cc = 0; cc < DH / 32; ++cc) {
-            uint32_t rr[32];
-            tmem_ld32(tO + 32 * cc, rr);
-            tmem_ld_wait();
+              for (int cc = 0; cc < DH / 32; ++cc) {
+                uint32_t rr[32];
+                tmem_ld32(tO + 32 * cc, rr);
+                tmem_ld_wait();
 #pragma unroll
-            for (int e = 0; e < 32; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
-            tmem_st32(tO + 32 * cc, rr);
-          }
-        }
-        if (valid < BKV) {
-          // last, partial key tile: clear the value rows past kv_len so stale
-          // (possibly non-finite) data cannot meet the zero probabilities (both
-          // groups write the same zeros: each must see them before its PV)
-          const int vsi = cv + j, vst = vsi % V_STAGES;
-          if (!__all_sync(0xffffffffu, mbar_wait(&v_full[vst], (vsi / V_STAGES) & 1, abort_flag, p.err))) {
-            ok = false;
-            break;
-          }
-          if (r >= valid) {
+                for (int e = 0; e < 32; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
+                tmem_st32(tO + 32 * cc, rr);
+              }
+            }
+            // ... and, on the last, partial key tile, clear the value rows past
+            // kv_len so stale (possibly non-finite) data cannot meet the zero
+            // probabilities (both groups write the same zeros: each must see
+            // them before its PV)
+            if (valid < BKV) {
+              const int vsi = cv + j, vst = vsi % V_STAGES;
+              if (!__all_sync(0xffffffffu, mbar_wait(&v_full[vst], (vsi / V_STAGES) & 1, abort_flag, p.err))) {
+                ok = false;
+                break;
+              }
+              if (r >= valid) {
 #pragma unroll
-            for (int pn = 0; pn < 2; ++pn) {
-              uint4* v = reinterpret_cast<uint4*>(smem + OFF_V + vst * TILE_BYTES + pn * PANEL + r * 128);
+                for (int pn = 0; pn < 2; ++pn) {
+                  uint4* v = reinterpret_cast<uint4*>(smem + OFF_V + vst * TILE_BYTES + pn * PANEL + r * 128);
 #pragma unroll
-              for (int e = 0; e < 8; ++e) v[e] = make_uint4(0, 0, 0, 0);
+                  for (int e = 0; e < 8; ++e) v[e] = make_uint4(0, 0, 0, 0);
+                }
+              }
+              fence_proxy_async_smem();
             }
           }
-          fence_proxy_async_smem();
+          tmem_st_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(hf == 0 ? &p_full[t] : &p_full2[t]);
         }
-        tmem_st_wait();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&p_full[t]);
+        if (!ok) break;
+        l = l * alpha + ((rs[0] + rs[1]) + (rs[2] + rs[3]));
       }
       if (!ok) break;
       if (!__all_sync(0xffffffffu, mbar_wait(&o_done[t], co & 1, abort_flag, p.err))) break;
