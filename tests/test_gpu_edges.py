@@ -32,6 +32,16 @@ def test_attention_query_tile_pair_boundaries(dt):
     _attention_case(dt, 2, 128, lens, lens, 1.0, 21)
 
 
+@pytest.mark.parametrize("dt", ["f16", "bf16"])
+def test_attention_probability_half_boundaries(dt):
+    # a round's PV is issued in two halves of 64 keys as the softmax releases
+    # them: last key tiles with 63, 64 and 65 valid keys (the second half empty,
+    # exactly full, or holding one key), and a kv_len short of the segment
+    lens = [64, 63, 65, 192, 191, 193, 300]
+    kv = [64, 63, 65, 192, 191, 193, 129]
+    _attention_case(dt, 2, 128, lens, kv, 1.0, 27)
+
+
 def test_attention_single_key_and_single_query_segments():
     lens = [1, 1, 129, 1]
     _attention_case("f16", 2, 128, lens, [1, 1, 1, 1], 1.0, 22)
