@@ -101,7 +101,10 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ x
 // sum of squares reduced across the warp, and the row scaled from registers.
 // Two blocks per SM (at most 128 registers): 16 resident warps keep enough
 // loads in flight (35194 x 4096 rows: 6.36 TB/s, against 5.4 for the
-// two-pass streaming kernel and 4.9 at one block per SM).
+// two-pass streaming kernel and 4.9 at one block per SM).  The gain vector g,
+// the same for every row, is staged once per block in shared memory (8 KB at
+// d = 4096); read from global memory per row, its loads were hoisted beside
+// the row's 64 registers and spilled.
 template <int IN, int OUT, int VPL>
 __global__ void __launch_bounds__(256, 2) rmsnorm_rows_kernel(const void* __restrict__ x, const void* __restrict__ g,
                                                            void* __restrict__ y, int M_cap, const int* M_dev, int d,
@@ -121,7 +124,9 @@ __global__ void __launch_bounds__(256, 2) rmsnorm_rows_kernel(const void* __rest
   const int nwarps = gridDim.x * 8;
   const int d8 = d / 8;
   const uint4* xv = reinterpret_cast<const uint4*>(x);
-  const uint4* gv = reinterpret_cast<const uint4*>(g);
+  __shared__ uint4 g_sh[32 * VPL];
+  for (int v = threadIdx.x; v < d8; v += blockDim.x) g_sh[v] = __ldg(reinterpret_cast<const uint4*>(g) + v);
+  __syncthreads();
   uint4* yv = reinterpret_cast<uint4*>(y);
   uint32_t nonfinite = 0;
   for (int row = blockIdx.x * 8 + warp; row < M; row += nwarps) {
@@ -132,13 +137,18 @@ __global__ void __launch_bounds__(256, 2) rmsnorm_rows_kernel(const void* __rest
       const int v = lane + 32 * i;
       raw[i] = v < d8 ? __ldg(xv + base8 + v) : make_uint4(0, 0, 0, 0);
     }
+    // the sum of squares unpacks through an opaque copy of each word, so the
+    // scaling below unpacks again instead of keeping 8 floats per vector live
+    // from here (that reuse needed 128 float registers and spilled)
     float ss = 0.f;
 #pragma unroll
     for (int i = 0; i < VPL; ++i) {
       const uint32_t w[4] = {raw[i].x, raw[i].y, raw[i].z, raw[i].w};
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
-        const float a = lo16(w[k], IN == kF16), b = hi16(w[k], IN == kF16);
+        uint32_t wc;
+        asm volatile("mov.b32 %0, %1;" : "=r"(wc) : "r"(w[k]));
+        const float a = lo16(wc, IN == kF16), b = hi16(wc, IN == kF16);
         ss = fmaf(a, a, ss);
         ss = fmaf(b, b, ss);
       }
@@ -150,7 +160,7 @@ __global__ void __launch_bounds__(256, 2) rmsnorm_rows_kernel(const void* __rest
     for (int i = 0; i < VPL; ++i) {
       const int v = lane + 32 * i;
       if (v < d8) {
-        const uint4 gq = gv[v];
+        const uint4 gq = g_sh[v];
         const uint32_t w[4] = {raw[i].x, raw[i].y, raw[i].z, raw[i].w};
         const uint32_t gw[4] = {gq.x, gq.y, gq.z, gq.w};
         uint32_t o[4];
